@@ -1,0 +1,438 @@
+#!/usr/bin/env python3
+"""Benchmark of the AGS optimizer step (one step = the reduction pass + the
+update pass over a whole parameter set) on GB300.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload resnet50]
+  python bench.py --impl reference ...   # the CPU oracle on the host cores
+
+Prints ONE JSON line.  `value` is parameters updated per second over the whole
+job, device-resident inputs; `e2e` is the same metric through the C ABI with
+the replica gradients copied in from pinned host memory and the step record and
+per-layer statistics copied back inside the timed region.  Under torchrun every
+rank runs its own replica step on its own GPU (no collective on the data path:
+one optimizer step has nothing to exchange once the K replicas are local), and
+the time is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "AGS optimizer steps/sec and params/sec; achieved HBM GB/s vs ~8 TB/s peak"
+UNIT = "params/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def _args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="resnet50")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--soak-s", type=float, default=1.0,
+                    help="untimed load before the timed steps, so clock samples see load")
+    ap.add_argument("--cpu-sample-s", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+# ---------------------------------------------------------------------------
+# bytes per parameter (fp32)
+# ---------------------------------------------------------------------------
+
+def pass1_bytes_per_param(K: int) -> int:
+    """Reduction pass: read K replicas, write the mean over replica 0 (K > 1)."""
+    return 4 * K + (4 if K > 1 else 0)
+
+
+def pass2_bytes_per_param(with_momentum=True) -> int:
+    """Update pass: read gbar, w, m; write w, m."""
+    return 20 if with_momentum else 12
+
+
+def step_min_bytes_per_param(K: int) -> int:
+    """Algorithmic minimum of one step: read K replicas, w, m; write w, m."""
+    return 4 * K + 16
+
+
+# ---------------------------------------------------------------------------
+# clocks (nvidia-smi sampled while the GPU is loaded)
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=5)
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for _, line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx = float(parts[1])
+            except ValueError:
+                continue
+            for name, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# ncu-measured DRAM traffic of the dominant kernel (committed summary)
+# ---------------------------------------------------------------------------
+
+def _kernel_source_sha() -> str:
+    path = os.path.join(ROOT, "paper_2603_18112_gb300", "csrc", "tula_ags.cu")
+    return hashlib.sha256(open(path, "rb").read()).hexdigest()[:16]
+
+
+def _ncu_traffic(kernel: str, workload: str, params: int):
+    """Bytes per launch from profiles/dram_traffic.txt if it was taken on the current
+    kernel source; scaled by parameters when the capture was a smaller case."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    sha = _kernel_source_sha()
+    for line in open(path):
+        f = line.split()
+        if len(f) >= 5 and not line.startswith("#") and f[0] == kernel and f[1] == workload \
+                and f[2] == sha:
+            captured_params = int(f[3])
+            return float(f[4]) * params / captured_params
+    return None
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(path))
+        return float(d["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline leg and --impl reference)
+# ---------------------------------------------------------------------------
+
+def _host_inputs(wl, frac=1.0):
+    import numpy as np
+    import torch
+
+    from paper_2603_18112_gb300 import workloads as W
+    pset = wl.pset
+    if frac < 1.0:
+        keep, tot = [], 0
+        budget = frac * pset.n_params
+        for s, k in zip(pset.shapes, pset.kinds):
+            if tot >= budget and keep:
+                break
+            keep.append((s, k))
+            tot += int(np.prod(s))
+        sub = W.ParamSet(pset.name + "-sample")
+        for s, k in keep:
+            sub.add(s, k)
+        pset = sub
+    buf = W.allocate(wl, "cpu", pset=pset)
+    torch.set_num_threads(max(1, os.cpu_count() or 1))
+    W.fill_state(buf, wl)
+    W.fill_grads(buf, wl, step=1)
+    w = W.to_numpy(buf.w)
+    m = W.to_numpy(buf.m)
+    g = [W.to_numpy(buf.g[k]) for k in range(wl.K)]
+    return pset, w, m, g
+
+
+def _oracle_steps(wl, w, m, g, steps):
+    import numpy as np
+
+    import oracle as O
+    hp = O.OracleHP(K=wl.K, s_max=wl.smax)
+    scale = np.ones(len(w), np.float32)
+    state = O.new_state()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        O.ags_step(w, m, g, wl.lr, wl.momentum, wl.weight_decay, hp, scale=scale, state=state)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(wl, budget_s):
+    """The oracle as it stands (single-threaded C) on the host: a bounded number of
+    full optimizer steps over the same parameter set."""
+    pset, w, m, g = _host_inputs(wl)
+    t1 = _oracle_steps(wl, w, m, g, 1)
+    steps = max(1, min(50, int(budget_s / max(t1, 1e-6))))
+    t = _oracle_steps(wl, w, m, g, steps)
+    return {"value": pset.n_params * steps / t, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{steps} full steps of the {wl.name} parameter set "
+                      f"({pset.n_params} params, {pset.n_tensors} tensors, K={wl.K}) on the host, "
+                      f"single-threaded C oracle"}
+
+
+def run_reference(args, wl):
+    ws, rank, _ = _dist()
+    if rank != 0:
+        return
+    pset_full = wl.pset
+    _, w, m, g = _host_inputs(wl)
+    t1 = _oracle_steps(wl, w, m, g, 1)
+    total = args.steps + args.warmup
+    frac = min(1.0, 120.0 / max(1e-9, total * t1))
+    if frac < 1.0:
+        pset, w, m, g = _host_inputs(wl, frac)
+    else:
+        pset = pset_full
+    _oracle_steps(wl, w, m, g, args.warmup)
+    t = _oracle_steps(wl, w, m, g, args.steps)
+    value = pset.n_params * args.steps / t
+    sample = (f"each step: the single-threaded C oracle over "
+              f"{'all' if frac >= 1.0 else 'the first'} {pset.n_tensors} tensors "
+              f"({pset.n_params} of {pset_full.n_params} params) of the {wl.name} set, K={wl.K}")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * t / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic", "config": _config(wl, pset_full),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def _config(wl, pset):
+    return {"workload": f"{wl.name} parameter set, K={wl.K} replica gradient buffers",
+            "params": pset.n_params, "tensors": pset.n_tensors, "K": wl.K,
+            "global_batch": None, "seq_len": None, "parallelism": "replicas only (1 step per GPU)",
+            "l2": "inputs larger than L2 (no flush): "
+                  f"{(4 * wl.K + 16) * pset.n_params / 1e9:.2f} GB touched per step vs 126 MB L2"}
+
+
+# ---------------------------------------------------------------------------
+# GPU timing
+# ---------------------------------------------------------------------------
+
+def run_ours(args, wl):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2603_18112_gb300 import build as B
+    from paper_2603_18112_gb300 import tula_ags as T
+    from paper_2603_18112_gb300 import workloads as W
+
+    ws, rank, local = _dist()
+    if ws > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    if not B.LIB.exists():
+        B.build()
+    T.lib()
+
+    pset = wl.pset
+    N = pset.n_params
+    K = wl.K
+    buf = W.allocate(wl, "cuda")
+    W.fill_state(buf, wl)
+    W.fill_grads(buf, wl, step=1)
+    stream = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    step = T.AGSOptimizerStep(buf.w, buf.g, buf.m, s_max=wl.smax)
+
+    def barrier():
+        if ws > 1:
+            dist.barrier()
+
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            step.step(wl.lr, wl.momentum, wl.weight_decay, refresh_scale=(i == 0), stream=stream)
+    stream.synchronize()
+
+    # per-step pass boundaries, recorded by the library on `stream`
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    with torch.cuda.stream(stream):
+        for trio in evs:
+            for e in trio:
+                e.record(stream)
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    # untimed load so the clock samples are taken under load (part of the warm-up)
+    soak = 0
+    t0 = time.time()
+    with torch.cuda.stream(stream):
+        while time.time() - t0 < args.soak_s:
+            for _ in range(20):
+                step.step(wl.lr, wl.momentum, wl.weight_decay, stream=stream)
+            soak += 20
+            stream.synchronize()
+    barrier()
+    torch.cuda.synchronize()
+    launches0 = T.tula_ags_launch_count()
+    with torch.cuda.stream(stream):
+        t_start.record(stream)
+        for trio in evs:
+            step.set_trace_events(trio)
+            step.step(wl.lr, wl.momentum, wl.weight_decay, stream=stream)
+        t_end.record(stream)
+    step.set_trace_events(None)
+    torch.cuda.synchronize()
+    barrier()
+    launches = T.tula_ags_launch_count() - launches0
+    clocks = sampler.stop()
+    elapsed_ms = t_start.elapsed_time(t_end)
+    p1 = [a.elapsed_time(b) for a, b, _ in evs]
+    p2 = [b.elapsed_time(c) for _, b, c in evs]
+
+    t_max_ms = elapsed_ms
+    if ws > 1:
+        tt = torch.tensor([elapsed_ms], dtype=torch.float64, device="cuda")
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        t_max_ms = float(tt.item())
+
+    # ---- end to end through the C ABI with host buffers -------------------
+    e2e = None
+    h2d = K * buf.total * 4
+    d2h = (T.TULA_STATE_LEN + T.TULA_STATS_LEN * pset.n_tensors) * 8
+    host_g = [torch.empty(buf.total, dtype=torch.float32, pin_memory=True) for _ in range(K)]
+    for k in range(K):
+        host_g[k].copy_(buf.g_flats[k][:buf.total])
+    host_state = torch.empty(T.TULA_STATE_LEN, dtype=torch.float64, pin_memory=True)
+    host_stats = torch.empty(pset.n_tensors, T.TULA_STATS_LEN, dtype=torch.float64,
+                             pin_memory=True)
+    torch.cuda.synchronize()
+    barrier()
+    e_start = torch.cuda.Event(enable_timing=True)
+    e_end = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e_start.record(stream)
+        for _ in range(args.e2e_steps):
+            for k in range(K):
+                buf.g_flats[k][:buf.total].copy_(host_g[k], non_blocking=True)
+            step.step(wl.lr, wl.momentum, wl.weight_decay, stream=stream)
+            host_state.copy_(step.state, non_blocking=True)
+            host_stats.copy_(step.stats, non_blocking=True)
+        e_end.record(stream)
+    stream.synchronize()
+    e2e_ms = e_start.elapsed_time(e_end)
+    if ws > 1:
+        tt = torch.tensor([e2e_ms], dtype=torch.float64, device="cuda")
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    e2e = {"value": ws * N * args.e2e_steps / (e2e_ms / 1e3), "unit": UNIT,
+           "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps}
+
+    if rank != 0:
+        dist.destroy_process_group()
+        return
+
+    peak, peak_kind = _peaks()
+    p1_avg_ms = statistics.fmean(p1)
+    p2_avg_ms = statistics.fmean(p2)
+    p1_bytes = pass1_bytes_per_param(K) * N
+    p2_bytes = pass2_bytes_per_param() * N
+    achieved = p1_bytes / (p1_avg_ms / 1e3) / 1e9
+    ms_per_step = t_max_ms / args.steps
+    step_gbs = step_min_bytes_per_param(K) * N / (ms_per_step / 1e3) / 1e9
+    traffic = _ncu_traffic("k_reduce", wl.name, N)
+    line = {
+        "metric": METRIC, "value": ws * N * args.steps / (t_max_ms / 1e3), "unit": UNIT,
+        "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+        "steps_per_s": 1e3 / ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": _config(wl, pset),
+        "roofline": {"bound": "hbm", "kernel": "k_reduce (replica mean + norms)",
+                     "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "peak_kind": peak_kind,
+                     "traffic": traffic, "bytes_per_launch": p1_bytes,
+                     "ms_per_launch": p1_avg_ms},
+        "update_pass": {"kernel": "k_update", "bytes_per_launch": p2_bytes,
+                        "ms_per_launch": p2_avg_ms,
+                        "achieved_gbs": p2_bytes / (p2_avg_ms / 1e3) / 1e9},
+        "step_hbm": {"algorithmic_bytes_per_param": step_min_bytes_per_param(K),
+                     "achieved_gbs": step_gbs, "frac": step_gbs / peak,
+                     "frac_of_8tbs": step_gbs / 8000.0},
+        "e2e": e2e,
+        "gpu_launches": launches,
+        "clocks": clocks,
+        "soak_steps": soak,
+    }
+    if not args.no_cpu_baseline and ws == 1:
+        line["cpu_baseline"] = cpu_baseline(wl, args.cpu_sample_s)
+    print(json.dumps(line), flush=True)
+    if ws > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = _args()
+    from paper_2603_18112_gb300 import workloads as W
+    wl = W.workload(args.workload)
+    if args.impl == "reference":
+        run_reference(args, wl)
+    else:
+        run_ours(args, wl)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,192 @@
+/*
+ * libtula_ags -- the data-parallel optimizer step of Adaptive Gradient
+ * Scaling (AGS) from Tula (arXiv 2603.18112), on one NVIDIA GB300 (sm_103a).
+ *
+ * One step, per the paper:
+ *   1. the mean of K replica gradient buffers (Eq. 1c: synchronous data-
+ *      parallel SGD averages the N workers' gradients; here the K replicas
+ *      sit in one GPU's HBM and the all-reduce becomes an in-place mean);
+ *   2. per-layer squared norms of the mean gradient (and of the weights);
+ *   3. the gradient-variability metric Delta(G) = |(|G_i|^2 - |G_{i-1}|^2) /
+ *      |G_{i-1}|^2| (Eq. 5) and the branch of Algorithm 1: scaled when
+ *      Delta < delta, unscaled (sensitive phase) otherwise;
+ *   4. the scaled update (Eq. 7b, Algorithm 1) applied through the wrapped
+ *      SGD optimizer with momentum and weight decay (Sec. IV-A, IV-B).
+ *
+ * Conventions for every entry point:
+ *   - Tensors are fp32, in caller-owned DEVICE memory, 4-byte aligned; the
+ *     fast path wants them 16-byte aligned (misaligned tensors take a scalar
+ *     path with the same results).
+ *   - Arrays of pointers (param_ptrs, grad_ptrs, ...) and numels are HOST
+ *     arrays, read during the call only.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = the legacy
+ *     default stream).  They allocate nothing, never synchronize the host,
+ *     and perform no host<->device copy, so they can be captured into a CUDA
+ *     graph.  Results are bitwise reproducible run to run, and independent of
+ *     the grid size (the reduction order depends on the numels only).
+ *   - The workspace is caller-owned device memory of at least
+ *     tula_ags_workspace_size() bytes, ZERO-FILLED before its first use; the
+ *     library leaves it re-usable (its counters back at zero) after every
+ *     call.  Calls that share a workspace must be ordered (one stream).
+ *   - Return value: TULA_OK (0) or a negative TULA_ERR_* code.  Argument
+ *     errors are detected on the host before anything is enqueued.
+ *   - Element-wise arithmetic is IEEE fp32, one rounding per operation, in the
+ *     order written below (no fused multiply-add).  Norms are fp64 sums of
+ *     fp32 partial sums of squares.
+ */
+#ifndef TULA_AGS_H
+#define TULA_AGS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define TULA_AGS_VERSION 1
+
+#define TULA_OK 0
+#define TULA_ERR_ARG (-1)         /* NULL where a pointer is required, n_tensors < 1, K outside
+                                     [1, TULA_MAX_K], numel < 0, unaligned fp32 pointer, bad enum,
+                                     mom_ptrs NULL with momentum != 0, refresh with K == 1 */
+#define TULA_ERR_WORKSPACE (-2)   /* workspace NULL or smaller than tula_ags_workspace_size() */
+#define TULA_ERR_CUDA (-3)        /* a kernel launch failed; see tula_ags_last_cuda_error() */
+#define TULA_ERR_UNSUPPORTED (-4) /* a valid but unimplemented combination of options */
+
+#define TULA_MAX_K 16
+
+/* How the per-tensor coefficient c_p on the gradient is chosen. */
+#define TULA_RULE_AGS 0    /* Algorithm 1: c_p = gradscale_p when Delta < delta, else 1 */
+#define TULA_RULE_NONE 1   /* vanilla large-batch training (LBT): c_p = 1 */
+#define TULA_RULE_LARS 2   /* prior art named in Sec. V-B: c_p = lars_trust * |w_p| / |g_p|,
+                              every step (1 when either norm is 0) */
+#define TULA_RULE_STATIC 3 /* static scaling U(s) of Eq. 8: c_p = static_s when Delta < delta */
+
+/* Granularity of gradscale (Algorithm 1 keeps one entry per parameter). */
+#define TULA_SCALE_PER_TENSOR 0  /* one factor per tensor: hp->scale[p] */
+#define TULA_SCALE_PER_ELEMENT 1 /* one factor per element: hp->scale_elem[p][j] */
+
+#define TULA_BRANCH_AUTO 0     /* Algorithm 1's test Delta < delta */
+#define TULA_BRANCH_SCALED 1   /* force the scaled branch (tests) */
+#define TULA_BRANCH_UNSCALED 2 /* force the unscaled branch (tests) */
+
+/* hp->state, device fp64 [TULA_STATE_LEN]; zero-filled = before the first step. */
+#define TULA_STATE_G2_PREV 0 /* |G_{i-1}|^2 of Eq. 5 (after a step: that step's |G|^2) */
+#define TULA_STATE_STEPS 1   /* steps done */
+#define TULA_STATE_DELTA 2   /* Delta of the last step (+inf at the first step) */
+#define TULA_STATE_SCALED 3  /* 1 if the last step took the scaled branch, else 0 */
+#define TULA_STATE_LEN 4
+
+/* Per-layer statistics rows, device fp64 [n_tensors][TULA_STATS_LEN]. */
+#define TULA_STAT_W_SQ 0      /* |w_p|^2 before the update */
+#define TULA_STAT_G_SQ 1      /* |gbar_p|^2, gbar = mean of the K replicas */
+#define TULA_STAT_G0_SQ 2     /* |g_{0,p}|^2, replica 0 before averaging */
+#define TULA_STAT_W_NORM 3    /* |w_p| */
+#define TULA_STAT_G_NORM 4    /* |gbar_p| */
+#define TULA_STAT_RATIO 5     /* |w_p| / |gbar_p| (LARS trust ratio), 0 when |gbar_p| = 0 */
+#define TULA_STAT_COEF 6      /* c_p applied to the gradient this step (NaN: per-element scale) */
+#define TULA_STAT_SCALE 7     /* gradscale_p after the step (0 without a per-tensor scale) */
+#define TULA_STATS_LEN 8
+
+typedef struct tula_ags_hparams {
+    int K;             /* replica gradient buffers, 1 .. TULA_MAX_K */
+    int rule;          /* TULA_RULE_* (default AGS) */
+    int granularity;   /* TULA_SCALE_* (default PER_TENSOR) */
+    int force_branch;  /* TULA_BRANCH_* (default AUTO) */
+    int refresh_scale; /* 1: after this step's update, run UpdateGradScale of Algorithm 1 with
+                          g_small = replica 0 (a sub-batch of the large batch, same weights) and
+                          g_large = the mean: gradscale_p = min(|g_0p| / (|gbar_p| + eps), s_max).
+                          Needs K > 1 and PER_TENSOR; the step itself uses the old gradscale. */
+    float delta;       /* threshold on Delta (default 0.5, Sec. III-C and IV-B) */
+    float eps;         /* stability term of UpdateGradScale (default 1e-8, Algorithm 1) */
+    float s_max;       /* bound on gradscale, sqrt(b_large / b_small) (default sqrt(K)) */
+    float static_s;    /* s of Eq. 8 for TULA_RULE_STATIC (default 1) */
+    float lars_trust;  /* trust coefficient for TULA_RULE_LARS (default 1) */
+    float *scale;                 /* device fp32 [n_tensors]: gradscale per tensor (AGS, PER_TENSOR);
+                                     written when refresh_scale is set */
+    float *const *scale_elem;     /* HOST array of n_tensors device fp32 pointers: gradscale per
+                                     element (AGS, PER_ELEMENT); read only when scaled */
+    double *state;                /* device fp64 [TULA_STATE_LEN], read and written */
+    double *layer_stats;          /* device fp64 [n_tensors][TULA_STATS_LEN], or NULL */
+    void *workspace;              /* device, >= tula_ags_workspace_size(), zero before first use */
+    size_t workspace_bytes;
+    int grid_ctas;                /* CTAs per launch; 0 = one wave of resident CTAs (results do
+                                     not depend on it) */
+    void *trace_events[3];        /* optional cudaEvent_t, recorded on `stream` before the
+                                     reduction pass, between the passes, after the update pass */
+} tula_ags_hparams;
+
+/* Fills *hp with the paper's defaults for K replicas: AGS, per tensor, automatic branch,
+ * delta 0.5, eps 1e-8, s_max sqrt(K) (b_small = one replica's share of the large batch),
+ * static_s 1, lars_trust 1; all pointers NULL, grid_ctas 0. */
+void tula_ags_default_hparams(tula_ags_hparams *hp, int K);
+
+/* Bytes of workspace needed for this list of tensor sizes (host only; K does not change it
+ * today and is validated). */
+int tula_ags_workspace_size(const int64_t *numels, int n_tensors, int K, size_t *bytes);
+
+/*
+ * One AGS optimizer step over n_tensors tensors (the whole model).
+ *   param_ptrs[p]          w_p, device fp32 [numels[p]], updated in place
+ *   grad_ptrs[k*n + p]     replica k of the gradient of tensor p, device fp32; when K > 1
+ *                          grad_ptrs[0*n + p] receives the mean gbar_p (an in-place all-reduce);
+ *                          the other replicas are only read
+ *   mom_ptrs[p]            momentum buffer m_p, device fp32, updated in place; mom_ptrs may be
+ *                          NULL only when momentum == 0 (then w <- w - lr * d)
+ *   numels[p] >= 0         element counts (0 = skipped)
+ * Per element, with c the coefficient of the rule (Algorithm 1, Eq. 8):
+ *   gbar = (((g_0 + g_1) + ...) + g_{K-1}) / K
+ *   d    = c * gbar + weight_decay * w
+ *   m    = momentum * m + d            (zero-filled m = torch.optim.SGD's first step)
+ *   w    = w - lr * m
+ * Also updates hp->state and, when given, hp->layer_stats and (refresh) hp->scale.
+ */
+int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mom_ptrs,
+                  const int64_t *numels, int n_tensors, float lr, float momentum,
+                  float weight_decay, const tula_ags_hparams *hp, void *stream);
+
+/*
+ * Per-layer statistics without an update (read-only on every tensor): rows of
+ * TULA_STATS_LEN fp64 as above, columns TULA_STAT_COEF and TULA_STAT_SCALE set to 0.
+ * grad_ptrs[k*n + p] as in tula_ags_step.  stats_out: device fp64 [n_tensors][8].
+ */
+int tula_layer_stats(const float *const *param_ptrs, const float *const *grad_ptrs, int K,
+                     const int64_t *numels, int n_tensors, double *stats_out, void *workspace,
+                     size_t workspace_bytes, void *stream);
+
+/*
+ * UpdateGradScale of Algorithm 1 from a small-batch gradient g_small[p] and the large-batch
+ * gradient g_large[p] (device fp32), with hp->eps and hp->s_max:
+ *   PER_TENSOR  (hp->scale[p]):       min(|g_small_p| / (|g_large_p| + eps), s_max), fp64, rounded
+ *   PER_ELEMENT (hp->scale_elem[p][j]): fminf(|g_small / (g_large + eps)|, s_max), fp32
+ * Uses hp->workspace (PER_TENSOR); hp->state is not touched.
+ */
+int tula_ags_update_scale(const float *const *g_small, const float *const *g_large,
+                          const int64_t *numels, int n_tensors, const tula_ags_hparams *hp,
+                          void *stream);
+
+/* Human-readable text for a TULA_* status code. */
+const char *tula_ags_error_string(int code);
+
+/* The cudaError_t of the last failed launch on this thread (0 if none). */
+int tula_ags_last_cuda_error(void);
+
+/* Number of kernels this process has launched through the library. */
+uint64_t tula_ags_launch_count(void);
+
+/*
+ * Host-only view of the work decomposition: tensor p is split into
+ * max(1, ceil(numels[p] / tula_ags_chunk_elems())) chunks; chunk_start_out[p] is the index of
+ * its first chunk and chunk_start_out[n_tensors] the total (n_tensors + 1 entries).
+ */
+int tula_ags_plan_chunks(const int64_t *numels, int n_tensors, int64_t *chunk_start_out);
+
+/* Elements per chunk (work item) of the reduction and update passes. */
+int tula_ags_chunk_elems(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TULA_AGS_H */

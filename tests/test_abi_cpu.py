@@ -1,0 +1,120 @@
+"""The C ABI on the host (no GPU): exports, defaults, workspace sizing, the chunk
+plan, and argument validation (which returns before any CUDA call)."""
+import ctypes
+import json
+import math
+import os
+
+import pytest
+
+from paper_2603_18112_gb300 import build as B
+from paper_2603_18112_gb300 import tula_ags as T
+from paper_2603_18112_gb300 import workloads as W
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "paper_hparams.json")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    B.build()
+    return T.lib()
+
+
+def test_every_declared_function_is_exported(lib):
+    names = T.header_functions()
+    assert "tula_ags_step" in names and "tula_layer_stats" in names
+    for name in names:
+        assert hasattr(lib, name), name
+
+
+def test_defaults_match_paper(lib):
+    gold = json.load(open(GOLDEN))
+    for K in (1, 4, 8, 16):
+        hp = T.tula_ags_default_hparams(K)
+        assert hp.K == K
+        assert hp.rule == T.TULA_RULE_AGS and hp.granularity == T.TULA_SCALE_PER_TENSOR
+        assert hp.delta == gold["delta"]["value"]
+        assert hp.eps == pytest.approx(gold["eps"]["value"], rel=1e-7)
+        assert hp.s_max == pytest.approx(math.sqrt(K), rel=1e-7)  # sqrt(b_large / b_small)
+        assert not hp.scale and not hp.state and not hp.workspace
+
+
+def test_plan_covers_every_element_once(lib):
+    C = T.tula_ags_chunk_elems()
+    numels = [0, 1, 3, C - 1, C, C + 1, 5 * C + 7, 64]
+    starts = T.tula_ags_plan_chunks(numels)
+    assert starts[0] == 0
+    for p, n in enumerate(numels):
+        nch = starts[p + 1] - starts[p]
+        assert nch == max(1, math.ceil(n / C))
+        covered = sum(min(C, n - i * C) for i in range(nch)) if n else 0
+        assert covered == n
+    assert starts == T.tula_ags_plan_chunks(numels)  # depends on the numels only
+
+
+def test_workspace_size_grows_with_chunks(lib):
+    ps = W.param_set("resnet50")
+    a = T.tula_ags_workspace_size(ps.numels, 8)
+    b = T.tula_ags_workspace_size(ps.numels + [10 ** 8], 8)
+    assert 0 < a < b and a % 256 == 0
+    assert T.tula_ags_workspace_size(ps.numels, 1) == a
+
+
+@pytest.mark.parametrize("numels,K", [([], 1), ([3, -1], 1), ([3], 0), ([3], 17)])
+def test_workspace_size_rejects(lib, numels, K):
+    with pytest.raises(T.TulaError) as e:
+        T.tula_ags_workspace_size(numels, K)
+    assert e.value.code == T.TULA_ERR_ARG
+
+
+def _call_step(lib, n=2, K=1, params=None, grads=None, moms=None, numels=None, hp=None,
+               momentum=0.9):
+    P = ctypes.c_void_p
+    fake = [0x10000 * (i + 1) for i in range(64)]  # aligned, never dereferenced on error paths
+    params = params if params is not None else fake[:n]
+    grads = grads if grads is not None else fake[8:8 + K * n]
+    numels = numels if numels is not None else [5] * n
+    pa = (P * max(1, len(params)))(*params)
+    ga = (P * max(1, len(grads)))(*grads)
+    ma = None if moms == "null" else (P * n)(*(moms or fake[40:40 + n]))
+    na = (ctypes.c_int64 * max(1, len(numels)))(*numels)
+    if hp is None:
+        hp = T.tula_ags_default_hparams(K)
+        hp.scale = 0x20000
+        hp.state = 0x30000
+        hp.workspace = 0x40000
+        hp.workspace_bytes = 1 << 30
+    return lib.tula_ags_step(pa, ga, ma, na, len(numels), 0.1, momentum, 0.0,
+                             ctypes.byref(hp), None)
+
+
+def test_step_argument_errors(lib):
+    assert _call_step(lib, numels=[]) == T.TULA_ERR_ARG                 # n_tensors < 1
+    assert _call_step(lib, numels=[5, -2]) == T.TULA_ERR_ARG           # negative numel
+    assert _call_step(lib, params=[0x10000, 0]) == T.TULA_ERR_ARG      # NULL param
+    assert _call_step(lib, params=[0x10000, 0x10002]) == T.TULA_ERR_ARG  # not 4-byte aligned
+    assert _call_step(lib, moms="null") == T.TULA_ERR_ARG              # momentum without buffer
+    hp = T.tula_ags_default_hparams(1)
+    assert _call_step(lib, hp=hp) == T.TULA_ERR_ARG                    # no state / scale
+    for field, bad in (("K", 0), ("K", 17), ("rule", 9), ("granularity", 5), ("force_branch", 7)):
+        hp = T.tula_ags_default_hparams(1)
+        hp.scale, hp.state, hp.workspace, hp.workspace_bytes = 0x20000, 0x30000, 0x40000, 1 << 30
+        setattr(hp, field, bad)
+        assert _call_step(lib, hp=hp) == T.TULA_ERR_ARG, field
+    hp = T.tula_ags_default_hparams(1)
+    hp.scale, hp.state, hp.workspace, hp.workspace_bytes = 0x20000, 0x30000, 0x40000, 1 << 30
+    hp.refresh_scale = 1                                                # K = 1 has no g_small
+    assert _call_step(lib, hp=hp) == T.TULA_ERR_ARG
+    hp = T.tula_ags_default_hparams(2)
+    hp.scale, hp.state, hp.workspace, hp.workspace_bytes = 0x20000, 0x30000, 0x40000, 16
+    assert _call_step(lib, K=2, hp=hp) == T.TULA_ERR_WORKSPACE          # too small
+    hp.workspace_bytes, hp.workspace = 1 << 30, 0x40010
+    assert _call_step(lib, K=2, hp=hp) == T.TULA_ERR_WORKSPACE          # not 256-byte aligned
+    hp.workspace = 0
+    assert _call_step(lib, K=2, hp=hp) == T.TULA_ERR_WORKSPACE
+
+
+def test_error_strings(lib):
+    for code in (0, -1, -2, -3, -4, 99):
+        assert isinstance(T.tula_ags_error_string(code), str)
+    assert T.tula_ags_last_cuda_error() == 0

@@ -1,0 +1,266 @@
+"""GPU parity: the CUDA library (through its C ABI) against the CPU oracle on the
+same seeded inputs, element by element, over multi-step runs that take both
+branches of Algorithm 1, at sizes that span many chunks and ragged tails and at
+the full sizes of the paper's parameter sets."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from _parity import (Pair, assert_f32_close, assert_norm_close, assert_state_close,
+                     assert_stats_close)
+from paper_2603_18112_gb300 import tula_ags as T
+from paper_2603_18112_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+CHUNK = 16384
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2603_18112_gb300 import build
+    build.build()
+    T.lib()
+
+
+def _ragged_pset(extra=()):
+    ps = W.ParamSet("ragged")
+    for n in (0, 1, 3, 4, 5, 63, 64, 65, 4095, CHUNK - 1, CHUNK, CHUNK + 1, 40000, 100003,
+              *extra):
+        ps.add((n,), W.KIND_NORMAL)
+    return ps
+
+
+def test_resnet20_ten_steps():
+    """ResNet-20 parameter set, K = 1, the 10-step multiplier schedule (both branches)."""
+    wl = W.workload("resnet20")
+    pair = Pair(wl)
+    W.fill_grads(pair.buf, wl, step=0)
+    small = torch.empty_like(pair.buf.g_flats[0])
+    W.fill_small(pair.buf, wl, small, step=0)
+    pair.refresh_from(small)
+    for i, mult in enumerate(W.STEP_MULTIPLIERS):
+        pair.step(i + 1, mult)
+    assert pair.flags[0] == 0 and 1 in pair.flags and pair.flags[3] == 0  # x2 jump: sensitive
+
+
+@pytest.mark.parametrize("K", [1, 2, 3, 4, 5, 8, 16])
+@pytest.mark.parametrize("shift", [0, 1])
+def test_ragged_shapes(K, shift):
+    """Tensors of 0..100003 elements (ragged chunk tails); shift=1 misaligns every tensor."""
+    wl = W.workload("stress_k4", seed=11 + K, factor_range=(1e-3, 1e1), zero_patterns=False)
+    pair = Pair(wl, K=K, align=1 if shift else 64, shift=shift, pset=_ragged_pset())
+    # draw 1 twice (Delta = 0: scaled), then x2 (Delta = 3: unscaled), then a fresh draw
+    for i, (seed_step, mult) in enumerate(((1, 1.0), (1, 1.0), (1, 2.0), (2, 1.0))):
+        pair.step(seed_step, mult, refresh=(K > 1 and i == 0))
+    assert pair.flags[:3] == [0, 1, 0]
+
+
+@pytest.mark.parametrize("name", ["resnet18", "resnet50", "vgg16"])
+def test_full_parameter_sets(name):
+    """Full-size ResNet-18 (K=4), ResNet-50 (K=8), VGG-16 (K=8): refresh, scaled, unscaled."""
+    wl = W.workload(name)
+    pair = Pair(wl)
+    for i, mult in enumerate((1.0, 1.0, 2.0)):
+        pair.step(1, mult, refresh=(i == 0))
+    assert pair.flags == [0, 1, 0]
+
+
+@pytest.mark.parametrize("rule,gran,mom", [
+    (T.TULA_RULE_NONE, T.TULA_SCALE_PER_TENSOR, True),
+    (T.TULA_RULE_LARS, T.TULA_SCALE_PER_TENSOR, True),
+    (T.TULA_RULE_STATIC, T.TULA_SCALE_PER_TENSOR, True),
+    (T.TULA_RULE_AGS, T.TULA_SCALE_PER_ELEMENT, True),
+    (T.TULA_RULE_AGS, T.TULA_SCALE_PER_TENSOR, False),
+])
+def test_rules(rule, gran, mom):
+    wl = W.workload("resnet20", seed=21)
+    pair = Pair(wl, K=2, rule=rule, granularity=gran, with_momentum=mom, static_s=4.0,
+                lars_trust=0.01, s_max=2.0)
+    for i, (seed_step, mult) in enumerate(((1, 1.0), (1, 1.0), (1, 2.0), (2, 1.0))):
+        pair.step(seed_step, mult, refresh=(gran == T.TULA_SCALE_PER_TENSOR and i == 0))
+    assert pair.flags[:3] == [0, 1, 0]
+
+
+def test_many_tensors_span_several_launches():
+    """1000 tensors with K = 16 need several parameter blocks per pass."""
+    rng = np.random.default_rng(5)
+    ps = W.ParamSet("many")
+    for n in rng.integers(1, 5000, size=1000):
+        ps.add((int(n),), W.KIND_NORMAL)
+    wl = W.workload("stress_k16", seed=31)
+    pair = Pair(wl, pset=ps)
+    before = T.tula_ags_launch_count()
+    for i, mult in enumerate((1.0, 1.0)):
+        pair.step(i + 1, mult, refresh=(i == 0))
+    assert T.tula_ags_launch_count() - before >= 2 * 2 * 2
+
+
+def test_zero_gradients_and_weights():
+    """All-zero gradients: |G|^2 = 0, the next step has Delta = inf/NaN -> unscaled."""
+    ps = _ragged_pset()
+    wl = W.workload("stress_k4", seed=41, factor_range=(0.0, 0.0))
+    wl = W.Workload(**{**wl.__dict__, "factor_range": None, "grad_std": 0.0, "w_std": 0.0})
+    pair = Pair(wl, K=4, pset=ps, rule=T.TULA_RULE_LARS)
+    pair.step(1, 1.0)
+    pair.step(2, 1.0)
+    st = pair.gpu.state.cpu().numpy()
+    assert st[0] == 0.0 and st[3] == 0.0
+    assert np.all(pair.gpu.stats.cpu().numpy()[:, T.TULA_STAT_COEF] == 1.0)
+
+
+def _inputs_snapshot(buf):
+    return ([f.clone() for f in buf.g_flats], buf.w_flat.clone(),
+            buf.m_flat.clone() if buf.m_flat is not None else None)
+
+
+def _restore(buf, snap):
+    for f, s in zip(buf.g_flats, snap[0]):
+        f.copy_(s)
+    buf.w_flat.copy_(snap[1])
+    if snap[2] is not None:
+        buf.m_flat.copy_(snap[2])
+
+
+@pytest.mark.parametrize("name", ["resnet18", "resnet50"])
+def test_bitwise_reproducible_across_runs_and_grids(name):
+    wl = W.workload(name)
+    buf = W.allocate(wl, "cuda")
+    W.fill_state(buf, wl)
+    W.fill_grads(buf, wl, step=1)
+    snap = _inputs_snapshot(buf)
+    outs = []
+    for grid in (0, 0, 1, 7, 333):
+        _restore(buf, snap)
+        st = T.AGSOptimizerStep(buf.w, buf.g, buf.m, grid_ctas=grid)
+        st.state.copy_(torch.tensor([1.0, 3.0, 0.0, 0.0], dtype=torch.float64))
+        st.step(wl.lr, wl.momentum, wl.weight_decay, refresh_scale=True)
+        torch.cuda.synchronize()
+        outs.append([buf.g_flats[0].clone(), buf.w_flat.clone(), buf.m_flat.clone(),
+                     st.stats.clone(), st.state.clone(), st.scale.clone()])
+    for o in outs[1:]:
+        for a, b in zip(outs[0], o):
+            assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("K", [1, 3, 4])
+def test_layer_stats(K):
+    wl = W.workload("resnet18", seed=51)
+    buf = W.allocate(wl, "cuda", K=K)
+    W.fill_state(buf, wl)
+    W.fill_grads(buf, wl, step=1)
+    g_before = [f.clone() for f in buf.g_flats]
+    ws = T.new_workspace(buf.numels, K)
+    stats = torch.zeros(buf.pset.n_tensors, 8, dtype=torch.float64, device="cuda")
+    T.tula_layer_stats(buf.w, buf.g, stats, ws)
+    ref = O.layer_stats(W.to_numpy(buf.w), [W.to_numpy(buf.g[k]) for k in range(K)])
+    torch.cuda.synchronize()
+    assert_stats_close(stats.cpu().numpy(), ref, "layer_stats")
+    for a, b in zip(g_before, buf.g_flats):
+        assert torch.equal(a, b)  # read-only
+
+
+@pytest.mark.parametrize("gran", [T.TULA_SCALE_PER_TENSOR, T.TULA_SCALE_PER_ELEMENT])
+def test_update_scale(gran):
+    wl = W.workload("resnet20", seed=61)
+    buf = W.allocate(wl, "cuda", K=2, pset=_ragged_pset(extra=(7, 300001)))
+    W.fill_grads(buf, wl, step=1)
+    gs, gl = buf.g[0], buf.g[1]
+    hp = T.tula_ags_default_hparams(4)
+    hp.granularity = gran
+    n = buf.pset.n_tensors
+    scale = torch.zeros(n, dtype=torch.float32, device="cuda")
+    ws = T.new_workspace(buf.numels, 1)
+    hp.scale, hp.workspace, hp.workspace_bytes = scale.data_ptr(), ws.data_ptr(), ws.numel()
+    se = [torch.zeros_like(t) for t in gs]
+    keep = None
+    if gran == T.TULA_SCALE_PER_ELEMENT:
+        keep = T._tensor_ptrs(se)
+        hp.scale_elem = T.ctypes.cast(keep, T.c_void_p).value
+    T.tula_ags_update_scale(gs, gl, hp)
+    ref_scale = np.zeros(n, np.float32)
+    ref_se = [np.zeros(t.numel(), np.float32) for t in gs]
+    O.update_scale(W.to_numpy(gs), W.to_numpy(gl), 1e-8, 2.0, gran, scale=ref_scale,
+                   scale_elem=ref_se)
+    torch.cuda.synchronize()
+    if gran == T.TULA_SCALE_PER_TENSOR:
+        assert_norm_close(scale.cpu().numpy(), ref_scale, "scale")
+    else:
+        for p in range(n):
+            assert np.array_equal(se[p].reshape(-1).cpu().numpy(), ref_se[p]), p
+
+
+def _oracle_g2(buf, K):
+    """|G|^2 of the replica mean over every tensor, one tensor at a time (oracle)."""
+    total = 0.0
+    for p in range(buf.pset.n_tensors):
+        g = [buf.g[k][p].reshape(-1).cpu().numpy() for k in range(K)]
+        total += O.sqnorm(O.replica_mean(g))
+    return total
+
+
+@pytest.mark.parametrize("name", ["stress_k1", "stress_k4", "stress_k16"])
+def test_stress_full_size_sampled(name):
+    """The ~1.65e9-element stress set at full size, in the benchmark's launch shape: |G|^2
+    against the oracle over every tensor; w, m, mean and statistics on 160 sampled tensors
+    (including the all-zero patterns and the largest tensor); a forced scaled second step."""
+    wl = W.workload(name)
+    K = wl.K
+    buf = W.allocate(wl, "cuda")
+    W.fill_state(buf, wl)
+    n = buf.pset.n_tensors
+    numels = buf.numels
+    rng = np.random.default_rng(9)
+    sample = sorted(set(rng.choice(n, 150, replace=False).tolist())
+                    | {7, 13, 21, 64 + 7, int(np.argmax(numels)), int(np.argmin(numels))})
+    gpu = T.AGSOptimizerStep(buf.w, buf.g, buf.m, s_max=wl.smax)
+    hp = O.OracleHP(K=K, s_max=wl.smax)
+    w_h = [buf.w[p].reshape(-1).cpu().numpy().copy() for p in sample]
+    m_h = [buf.m[p].reshape(-1).cpu().numpy().copy() for p in sample]
+    scale_h = np.ones(len(sample), np.float32)
+    if K == 1:
+        W.fill_grads(buf, wl, step=0)
+        small = torch.empty_like(buf.g_flats[0])
+        W.fill_small(buf, wl, small, step=0)
+        views = W._views(small, buf.offsets, buf.pset.shapes, numels)
+        T.tula_ags_update_scale(views, buf.g[0], gpu.hp)
+        O.update_scale([views[p].reshape(-1).cpu().numpy() for p in sample],
+                       [buf.g[0][p].reshape(-1).cpu().numpy() for p in sample], hp.eps,
+                       wl.smax, O.GRAN_TENSOR, scale=scale_h)
+        del small, views
+    for step, force in ((1, O.BRANCH_AUTO), (2, O.BRANCH_SCALED)):
+        W.fill_grads(buf, wl, step=step)
+        g_h = [[buf.g[k][p].reshape(-1).cpu().numpy().copy() for p in sample] for k in range(K)]
+        g2 = _oracle_g2(buf, K) if step == 1 else None
+        gpu.hp.force_branch = force
+        gpu.step(wl.lr, wl.momentum, wl.weight_decay, refresh_scale=(K > 1 and step == 1))
+        hp.force_branch = force if step == 2 else O.BRANCH_AUTO
+        hp.refresh_scale = K > 1 and step == 1
+        st_h = O.new_state()
+        stats_h = O.ags_step(w_h, m_h, g_h, wl.lr, wl.momentum, wl.weight_decay, hp,
+                             scale=scale_h, state=st_h)
+        torch.cuda.synchronize()
+        state = gpu.state.cpu().numpy()
+        stats = gpu.stats.cpu().numpy()
+        if step == 1:
+            assert_state_close(state, np.array([g2, 1.0, math.inf, 0.0]), name)
+            g2_prev = state[0]
+        else:
+            assert state[3] == 1.0
+            assert state[2] == pytest.approx(abs((state[0] - g2_prev) / g2_prev), rel=1e-12)
+            # |G|^2 is the fixed-order sum of the per-layer |gbar|^2
+            assert state[0] == pytest.approx(float(np.sum(stats[:, T.TULA_STAT_G_SQ])), rel=1e-12)
+        for i, p in enumerate(sample):
+            where = f"{name} step {step} tensor {p}"
+            if K > 1:
+                assert np.array_equal(buf.g[0][p].reshape(-1).cpu().numpy(), g_h[0][i]), where
+            assert_f32_close(buf.w[p].reshape(-1).cpu().numpy(), w_h[i], where + " w")
+            assert_f32_close(buf.m[p].reshape(-1).cpu().numpy(), m_h[i], where + " m")
+            for c in (0, 1, 2, 3, 4, 5, 6, 7):
+                assert_norm_close(stats[p, c:c + 1], stats_h[i, c:c + 1], f"{where} stat {c}")
+        assert_norm_close(gpu.scale.cpu().numpy()[sample], scale_h, name + " scale")
+    del buf, gpu
+    torch.cuda.empty_cache()
