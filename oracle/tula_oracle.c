@@ -13,9 +13,9 @@
  * Precision (a reading; the paper names none): parameters, gradients and
  * momentum are fp32 tensors, so every element-wise operation is one IEEE fp32
  * operation, in the order the equations write it, with no fused multiply-add
- * (build with -ffp-contract=off).  Squared norms, the global norm and the
- * variability metric are accumulated in fp64, sequentially, element 0 first;
- * the square of an fp32 value is exact in fp64.
+ * (build with -ffp-contract=off).  Squared norms are accumulated in fp64,
+ * element 0 first, with compensated summation (the square of an fp32 value is
+ * exact in fp64); the global norm and the variability metric are fp64.
  */
 #include <math.h>
 #include <stddef.h>
@@ -64,16 +64,26 @@ void oracle_replica_mean(const float *const *g, int K, int64_t n, float *out)
     }
 }
 
-/* Squared L2 norm |x|^2, fp64, sequential (the quantity |G|^2 of Eq. 5 is the
- * sum of these over all tensors). */
+/* Squared L2 norm |x|^2 (the quantity |G|^2 of Eq. 5 is the sum of these over
+ * all tensors).  Each square is exact in fp64; the squares are added in order,
+ * element 0 first, with Neumaier's compensated summation, so the result is the
+ * exact sum to within about two fp64 roundings whatever n is.  (A per-tensor
+ * scale or trust ratio rounds a ratio of these to fp32; an accurate sum keeps
+ * that rounding a property of the data, not of the summation order.) */
 double oracle_sqnorm(const float *x, int64_t n)
 {
-    double s = 0.0;
+    double s = 0.0, c = 0.0;
     for (int64_t j = 0; j < n; ++j) {
         double v = (double)x[j];
-        s = s + v * v;
+        double t = v * v;
+        double u = s + t;
+        if (fabs(s) >= fabs(t))
+            c = c + ((s - u) + t);
+        else
+            c = c + ((t - u) + s);
+        s = u;
     }
-    return s;
+    return s + c;
 }
 
 /* Eq. 5: Delta(G^(i)) = | (|G^(i)|^2 - |G^(i-1)|^2) / |G^(i-1)|^2 |.

@@ -93,7 +93,16 @@ def test_sqnorm_brute_force(n):
     x = (rng.standard_normal(n) * 10.0 ** rng.uniform(-6, 6, n)).astype(np.float32)
     exact = math.fsum(float(v) * float(v) for v in x)  # squares exact in fp64; fsum exact
     got = O.sqnorm(x)
-    assert abs(got - exact) <= max(n, 1) * 2.0 ** -53 * exact + 0.0
+    # compensated summation: within ~2 fp64 roundings of the exact sum, independent of n
+    assert abs(got - exact) <= 4 * 2.0 ** -53 * exact + 0.0
+
+
+def test_sqnorm_accuracy_independent_of_length():
+    rng = np.random.default_rng(99)
+    x = (rng.standard_normal(2_000_000) * 10.0 ** rng.uniform(-3, 3, 2_000_000)).astype(np.float32)
+    xs = x.astype(np.float64)
+    exact = math.fsum((xs * xs).tolist())
+    assert abs(O.sqnorm(x) - exact) <= 4 * 2.0 ** -53 * exact
 
 
 def test_sqnorm_closed_forms():
