@@ -102,6 +102,15 @@ __device__ __forceinline__ float sq4(float acc, float4 v) {
     return acc;
 }
 
+// fp64 sum of exact squares (an fp32 square is exact in fp64), one DFMA per term
+__device__ __forceinline__ double dsq4(double acc, float4 v) {
+    acc = __fma_rn((double)v.x, (double)v.x, acc);
+    acc = __fma_rn((double)v.y, (double)v.y, acc);
+    acc = __fma_rn((double)v.z, (double)v.z, acc);
+    acc = __fma_rn((double)v.w, (double)v.w, acc);
+    return acc;
+}
+
 __device__ __forceinline__ float4 add4(float4 a, float4 b) {
     return make_float4(__fadd_rn(a.x, b.x), __fadd_rn(a.y, b.y), __fadd_rn(a.z, b.z),
                        __fadd_rn(a.w, b.w));
@@ -257,7 +266,12 @@ __device__ void finalize(const Scalars &sc, double (*red)[kWarps]) {
 //
 // Template: KT = replicas known at compile time (0: runtime K <= 16);
 // WM = write the mean over replica 0; RW = also reduce |w|^2;
-// SS = g_small is a separate stream (role KS + 1) instead of replica 0.
+// SS = g_small is a separate stream (role KS + 1) instead of replica 0;
+// PR = precise norms: every exact fp64 square is added in fp64 (relative error
+// ~1e-15), for norms that feed a per-tensor coefficient (UpdateGradScale, LARS);
+// otherwise each thread sums <= 16 squares in fp32 before one fp64 add (~1e-7),
+// which is what the variability metric and the statistics need, at a fraction
+// of GB300's FP64 rate.
 // Pointer roles per tensor: [0, K) replicas, KS = w, KS + 1 = g_small.
 
 template <int KT>
@@ -266,7 +280,7 @@ struct P1 {
     static constexpr int NP = KS + 2;
 };
 
-template <int KT, bool WM, bool RW, bool SS>
+template <int KT, bool WM, bool RW, bool SS, bool PR>
 __device__ __forceinline__ void reduce_vec(const Table<P1<KT>::NP> &tab, int t, long long begin,
                                            int nv, const Scalars &sc, double &ag, double &as,
                                            double &aw) {
@@ -309,16 +323,24 @@ __device__ __forceinline__ void reduce_vec(const Table<P1<KT>::NP> &tab, int t, 
                 if (K > 1) {
                     s = mean4(s, sc);
                     if (WM) st_keep(out + 4 * (size_t)v, s);
-                    ps = sq4(ps, x[u][0]);
+                    if (PR) as = dsq4(as, x[u][0]); else ps = sq4(ps, x[u][0]);
                 }
-                pg = sq4(pg, s);
-                if (SS) ps = sq4(ps, sv[u]);
-                if (RW) pw = sq4(pw, wv[u]);
+                if (PR) {
+                    ag = dsq4(ag, s);
+                    if (SS) as = dsq4(as, sv[u]);
+                    if (RW) aw = dsq4(aw, wv[u]);
+                } else {
+                    pg = sq4(pg, s);
+                    if (SS) ps = sq4(ps, sv[u]);
+                    if (RW) pw = sq4(pw, wv[u]);
+                }
             }
         }
-        ag = __dadd_rn(ag, (double)pg);
-        if (K > 1 || SS) as = __dadd_rn(as, (double)ps);
-        if (RW) aw = __dadd_rn(aw, (double)pw);
+        if (!PR) {
+            ag = __dadd_rn(ag, (double)pg);
+            if (K > 1 || SS) as = __dadd_rn(as, (double)ps);
+            if (RW) aw = __dadd_rn(aw, (double)pw);
+        }
     }
 }
 
@@ -338,21 +360,21 @@ __device__ __forceinline__ void reduce_scalar(const Table<P1<KT>::NP> &tab, int 
         if (K > 1) {
             s = mean1(s, sc);
             if (WM) const_cast<float *>(tab.ptr[t][0])[j] = s;
-            as = __dadd_rn(as, (double)__fmul_rn(x0, x0));
+            as = __fma_rn((double)x0, (double)x0, as);
         }
-        ag = __dadd_rn(ag, (double)__fmul_rn(s, s));
+        ag = __fma_rn((double)s, (double)s, ag);
         if (SS) {
-            float y = __ldcs(tab.ptr[t][KS + 1] + j);
-            as = __dadd_rn(as, (double)__fmul_rn(y, y));
+            const double y = __ldcs(tab.ptr[t][KS + 1] + j);
+            as = __fma_rn(y, y, as);
         }
         if (RW) {
-            float y = __ldcs(tab.ptr[t][KS] + j);
-            aw = __dadd_rn(aw, (double)__fmul_rn(y, y));
+            const double y = __ldcs(tab.ptr[t][KS] + j);
+            aw = __fma_rn(y, y, aw);
         }
     }
 }
 
-template <int KT, bool WM, bool RW, bool SS>
+template <int KT, bool WM, bool RW, bool SS, bool PR>
 __global__ void __launch_bounds__(kThreads, 2)
     k_reduce(const __grid_constant__ Table<P1<KT>::NP> tab, const __grid_constant__ Scalars sc) {
     constexpr int KS = P1<KT>::KS;
@@ -374,7 +396,7 @@ __global__ void __launch_bounds__(kThreads, 2)
             if (SS) al |= reinterpret_cast<uintptr_t>(tab.ptr[t][KS + 1]);
             const int nv = (al & 15u) == 0 ? (int)((end - begin) >> 2) : 0;
             if (nv > 0)
-                reduce_vec<KT, WM, RW, SS>(tab, t, begin, nv, sc, acc[0], acc[1], acc[2]);
+                reduce_vec<KT, WM, RW, SS, PR>(tab, t, begin, nv, sc, acc[0], acc[1], acc[2]);
             reduce_scalar<KT, WM, RW, SS>(tab, t, begin + 4 * (long long)nv, end, sc, acc[0],
                                           acc[1], acc[2]);
         }
@@ -725,22 +747,22 @@ Scalars make_scalars(const tula_ags_hparams *hp, int K, int n, void *ws, const W
 }
 
 // Pass-1 dispatch over the compile-time replica count.
-template <int KT, bool WM, bool RW, bool SS, typename Fill>
+template <int KT, bool WM, bool RW, bool SS, bool PR, typename Fill>
 int run_reduce_k(int n, const int64_t *numels, const Scalars &sc, int grid, cudaStream_t s,
                  Fill fill) {
-    return launch_groups<P1<KT>::NP>(k_reduce<KT, WM, RW, SS>, n, numels, sc, grid, s, fill);
+    return launch_groups<P1<KT>::NP>(k_reduce<KT, WM, RW, SS, PR>, n, numels, sc, grid, s, fill);
 }
 
-template <bool WM, bool RW, bool SS, typename Fill>
+template <bool WM, bool RW, bool SS, bool PR, typename Fill>
 int run_reduce(int K, int n, const int64_t *numels, const Scalars &sc, int grid, cudaStream_t s,
                Fill fill) {
     switch (K) {
-    case 1: return run_reduce_k<1, false, RW, SS>(n, numels, sc, grid, s, fill);
-    case 2: return run_reduce_k<2, WM, RW, SS>(n, numels, sc, grid, s, fill);
-    case 4: return run_reduce_k<4, WM, RW, SS>(n, numels, sc, grid, s, fill);
-    case 8: return run_reduce_k<8, WM, RW, SS>(n, numels, sc, grid, s, fill);
-    case 16: return run_reduce_k<16, WM, RW, SS>(n, numels, sc, grid, s, fill);
-    default: return run_reduce_k<0, WM, RW, SS>(n, numels, sc, grid, s, fill);
+    case 1: return run_reduce_k<1, false, RW, SS, PR>(n, numels, sc, grid, s, fill);
+    case 2: return run_reduce_k<2, WM, RW, SS, PR>(n, numels, sc, grid, s, fill);
+    case 4: return run_reduce_k<4, WM, RW, SS, PR>(n, numels, sc, grid, s, fill);
+    case 8: return run_reduce_k<8, WM, RW, SS, PR>(n, numels, sc, grid, s, fill);
+    case 16: return run_reduce_k<16, WM, RW, SS, PR>(n, numels, sc, grid, s, fill);
+    default: return run_reduce_k<0, WM, RW, SS, PR>(n, numels, sc, grid, s, fill);
     }
 }
 
@@ -851,8 +873,13 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
         dst[KS + 1] = nullptr;
     };
     record(hp->trace_events[0], s);
-    rc = lars ? run_reduce<true, true, false>(K, n, numels, sc, hp->grid_ctas, s, fill1)
-              : run_reduce<true, false, false>(K, n, numels, sc, hp->grid_ctas, s, fill1);
+    // Norms feeding a coefficient (LARS, UpdateGradScale) are taken precisely.
+    if (lars)
+        rc = run_reduce<true, true, false, true>(K, n, numels, sc, hp->grid_ctas, s, fill1);
+    else if (hp->refresh_scale)
+        rc = run_reduce<true, false, false, true>(K, n, numels, sc, hp->grid_ctas, s, fill1);
+    else
+        rc = run_reduce<true, false, false, false>(K, n, numels, sc, hp->grid_ctas, s, fill1);
     if (rc) return rc;
     record(hp->trace_events[1], s);
 
@@ -907,7 +934,7 @@ int tula_layer_stats(const float *const *param_ptrs, const float *const *grad_pt
         dst[KS] = param_ptrs[p];
         dst[KS + 1] = nullptr;
     };
-    return run_reduce<false, true, false>(K, n, numels, sc, 0,
+    return run_reduce<false, true, false, false>(K, n, numels, sc, 0,
                                           static_cast<cudaStream_t>(stream), fill);
 }
 
@@ -949,7 +976,7 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
         dst[1] = nullptr;
         dst[2] = g_small[p];
     };
-    return run_reduce_k<1, false, false, true>(n, numels, sc, hp->grid_ctas, s, fill);
+    return run_reduce_k<1, false, false, true, true>(n, numels, sc, hp->grid_ctas, s, fill);
 }
 
 const char *tula_ags_error_string(int code) {
