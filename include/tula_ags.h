@@ -53,6 +53,8 @@ extern "C" {
 #define TULA_ERR_WORKSPACE (-2)   /* workspace NULL or smaller than tula_ags_workspace_size() */
 #define TULA_ERR_CUDA (-3)        /* a kernel launch failed; see tula_ags_last_cuda_error() */
 #define TULA_ERR_UNSUPPORTED (-4) /* a valid but unimplemented combination of options */
+#define TULA_ERR_SCRATCH_LIMIT (-5) /* tula_ags_step_static_scratch: the tensor list needs more
+                                       scratch than TULA_STATIC_SCRATCH_BYTES */
 
 #define TULA_MAX_K 16
 
@@ -165,6 +167,39 @@ int tula_layer_stats(const float *const *param_ptrs, const float *const *grad_pt
 int tula_ags_update_scale(const float *const *g_small, const float *const *g_large,
                           const int64_t *numels, int n_tensors, const tula_ags_hparams *hp,
                           void *stream);
+
+/*
+ * tula_ags_step_static_scratch -- the same optimizer step as tula_ags_step, for callers that
+ * cannot allocate device memory. (The paper has no counterpart; this is a deployment aid.)
+ *
+ * Who needs it: code that runs inside a host framework which owns every device allocation and
+ * forbids foreign ones, code on a latency-critical path where cudaMalloc's implicit device-wide
+ * synchronization is not acceptable, and plain C callers whose fixed call signature leaves no
+ * place to keep a workspace between calls.  Such a caller still passes every input and output
+ * (tensors, hp->scale, hp->state, hp->layer_stats); only the scratch moves.
+ *
+ * The scratch that tula_ags_step takes from hp->workspace (chunk partial sums, per-tensor sums,
+ * counters, coefficients) lives instead in one file-scope __device__ array of
+ * TULA_STATIC_SCRATCH_BYTES (4 MiB) inside this library.  Every GPU that loads the library holds
+ * that array until the process exits.  hp->workspace and hp->workspace_bytes are ignored.
+ *
+ * Limit: the scratch a tensor list needs is about 44 bytes per tensor plus 24 bytes per chunk of
+ * tula_ags_chunk_elems() elements (e.g. 4096 tensors and up to ~2.7e9 parameters).  A larger list
+ * is rejected with TULA_ERR_SCRATCH_LIMIT before anything is enqueued.
+ *
+ * Set-up: the first call on each device, with that device current, looks up the array's device
+ * address (cudaGetSymbolAddress); make that first call before any stream capture.
+ * Sharing: every call on a device uses the same array.  Each call clears the counters it needs
+ * zeroed (an asynchronous memset on `stream`) and otherwise overwrites what the previous call
+ * left, so calls that overlap on the GPU (different streams, or different host threads) race
+ * and must not be issued.  Allocates nothing: no cudaMalloc, no cudaFree, no allocating library
+ * call.  Arguments, semantics and other status codes are those of tula_ags_step.
+ */
+#define TULA_STATIC_SCRATCH_BYTES (4u << 20)
+int tula_ags_step_static_scratch(float *const *param_ptrs, float *const *grad_ptrs,
+                                 float *const *mom_ptrs, const int64_t *numels, int n_tensors,
+                                 float lr, float momentum, float weight_decay,
+                                 const tula_ags_hparams *hp, void *stream);
 
 /* Human-readable text for a TULA_* status code. */
 const char *tula_ags_error_string(int code);

@@ -986,6 +986,9 @@ const char *tula_ags_error_string(int code) {
     case TULA_ERR_WORKSPACE: return "workspace missing, too small or not 256-byte aligned";
     case TULA_ERR_CUDA: return "CUDA launch failed";
     case TULA_ERR_UNSUPPORTED: return "unsupported combination of options";
+    case TULA_ERR_SCRATCH_LIMIT:
+        return "tensor list needs more than the library's static scratch "
+               "(TULA_STATIC_SCRATCH_BYTES); use tula_ags_step with a workspace";
     default: return "unknown status";
     }
 }
@@ -995,3 +998,72 @@ int tula_ags_last_cuda_error(void) { return g_last_cuda; }
 uint64_t tula_ags_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 }  // extern "C"
+
+// ============================================================================
+// Allocation-free step: the scratch in a static device array
+// ============================================================================
+// For callers that cannot allocate device memory (see the header).  The step
+// itself is tula_ags_step; only where its scratch lives differs.
+
+namespace {
+
+constexpr size_t kStaticScratchBytes = TULA_STATIC_SCRATCH_BYTES;
+constexpr int kMaxDevices = 64;
+
+// One copy per device, alive until the process exits.  In host code this name
+// is only a handle: its device address comes from cudaGetSymbolAddress.
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+std::mutex g_static_mu;
+void *g_static_ptr[kMaxDevices] = {};
+
+// Device address of g_static_scratch on the current device, looked up once per device.
+int static_scratch_address(void **out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) {
+        g_last_cuda = (int)e;
+        return TULA_ERR_CUDA;
+    }
+    if (dev < 0 || dev >= kMaxDevices) return TULA_ERR_UNSUPPORTED;
+    std::lock_guard<std::mutex> lock(g_static_mu);
+    if (!g_static_ptr[dev]) {
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_static_scratch);
+        if (e != cudaSuccess || !p) {
+            g_last_cuda = (int)e;
+            return TULA_ERR_CUDA;
+        }
+        g_static_ptr[dev] = p;
+    }
+    *out = g_static_ptr[dev];
+    return TULA_OK;
+}
+
+}  // namespace
+
+extern "C" int tula_ags_step_static_scratch(float *const *param_ptrs, float *const *grad_ptrs,
+                                            float *const *mom_ptrs, const int64_t *numels,
+                                            int n_tensors, float lr, float momentum,
+                                            float weight_decay, const tula_ags_hparams *hp,
+                                            void *stream) {
+    long long nch = 0;
+    if (!hp || !valid_numels(numels, n_tensors, &nch)) return TULA_ERR_ARG;
+    const WsLayout L = ws_layout(n_tensors, nch);
+    if (L.total > kStaticScratchBytes) return TULA_ERR_SCRATCH_LIMIT;
+    void *scratch = nullptr;
+    int rc = static_scratch_address(&scratch);
+    if (rc) return rc;
+    // The array keeps the last call's contents: zero the tickets, done counter and
+    // branch flag (they precede the partial sums) before this call's kernels.
+    cudaError_t e = cudaMemsetAsync(scratch, 0, L.partials, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) {
+        g_last_cuda = (int)e;
+        return TULA_ERR_CUDA;
+    }
+    tula_ags_hparams local = *hp;
+    local.workspace = scratch;
+    local.workspace_bytes = kStaticScratchBytes;
+    return tula_ags_step(param_ptrs, grad_ptrs, mom_ptrs, numels, n_tensors, lr, momentum,
+                         weight_decay, &local, stream);
+}

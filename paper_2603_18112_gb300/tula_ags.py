@@ -19,6 +19,8 @@ from .build import HEADER, LIB
 c_int, c_float, c_void_p, c_size_t = ctypes.c_int, ctypes.c_float, ctypes.c_void_p, ctypes.c_size_t
 
 TULA_OK, TULA_ERR_ARG, TULA_ERR_WORKSPACE, TULA_ERR_CUDA, TULA_ERR_UNSUPPORTED = 0, -1, -2, -3, -4
+TULA_ERR_SCRATCH_LIMIT = -5
+TULA_STATIC_SCRATCH_BYTES = 4 << 20
 TULA_MAX_K = 16
 TULA_RULE_AGS, TULA_RULE_NONE, TULA_RULE_LARS, TULA_RULE_STATIC = 0, 1, 2, 3
 TULA_SCALE_PER_TENSOR, TULA_SCALE_PER_ELEMENT = 0, 1
@@ -76,6 +78,8 @@ def lib() -> ctypes.CDLL:
     L.tula_layer_stats.argtypes = [pp, pp, c_int, i64p, c_int, c_void_p, c_void_p, c_size_t,
                                    c_void_p]
     L.tula_ags_update_scale.argtypes = [pp, pp, i64p, c_int, hpp, c_void_p]
+    L.tula_ags_step_static_scratch.argtypes = [pp, pp, pp, i64p, c_int, c_float, c_float,
+                                               c_float, hpp, c_void_p]
     L.tula_ags_error_string.argtypes = [c_int]
     L.tula_ags_error_string.restype = ctypes.c_char_p
     L.tula_ags_last_cuda_error.restype = c_int
@@ -83,7 +87,7 @@ def lib() -> ctypes.CDLL:
     L.tula_ags_plan_chunks.argtypes = [i64p, c_int, i64p]
     L.tula_ags_chunk_elems.restype = c_int
     for name in ("tula_ags_workspace_size", "tula_ags_step", "tula_layer_stats",
-                 "tula_ags_update_scale", "tula_ags_plan_chunks"):
+                 "tula_ags_update_scale", "tula_ags_plan_chunks", "tula_ags_step_static_scratch"):
         getattr(L, name).restype = c_int
     _lib = L
     return L
@@ -192,6 +196,20 @@ def tula_ags_step(params, grads, moms, lr, momentum, weight_decay, hp: tula_ags_
                              _tensor_ptrs(moms) if moms is not None else None, _numels(params), n,
                              lr, momentum, weight_decay, ctypes.byref(hp), _stream_ptr(stream))
     _check(rc, "tula_ags_step")
+
+
+def tula_ags_step_static_scratch(params, grads, moms, lr, momentum, weight_decay,
+                                 hp: tula_ags_hparams, stream=None) -> None:
+    """tula_ags_step for callers that cannot allocate device memory: the step's scratch is
+    the library's static device array (hp.workspace is ignored).  Calls on one device must not
+    overlap on the GPU; make the first call on a device before any stream capture."""
+    n = len(params)
+    K = len(grads)
+    flat = [grads[k][p] for k in range(K) for p in range(n)]
+    rc = lib().tula_ags_step_static_scratch(
+        _tensor_ptrs(params), _tensor_ptrs(flat), _tensor_ptrs(moms) if moms is not None else None,
+        _numels(params), n, lr, momentum, weight_decay, ctypes.byref(hp), _stream_ptr(stream))
+    _check(rc, "tula_ags_step_static_scratch")
 
 
 def tula_layer_stats(params, grads, stats_out: torch.Tensor, workspace: torch.Tensor,
