@@ -180,12 +180,12 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
  *
  * The scratch that tula_ags_step takes from hp->workspace (chunk partial sums, per-tensor sums,
  * counters, coefficients) lives instead in one file-scope __device__ array of
- * TULA_STATIC_SCRATCH_BYTES (4 MiB) inside this library.  Every GPU that loads the library holds
+ * TULA_STATIC_SCRATCH_BYTES (16 MiB) inside this library.  Every GPU that loads the library holds
  * that array until the process exits.  hp->workspace and hp->workspace_bytes are ignored.
  *
- * Limit: the scratch a tensor list needs is about 44 bytes per tensor plus 24 bytes per chunk of
- * tula_ags_chunk_elems() elements (e.g. 4096 tensors and up to ~2.7e9 parameters).  A larger list
- * is rejected with TULA_ERR_SCRATCH_LIMIT before anything is enqueued.
+ * Limit: the scratch a tensor list needs (tula_ags_workspace_size) is about 100 bytes per tensor
+ * plus 6.1 bytes per 1000 parameters, e.g. 4096 tensors holding up to ~2.6e9 parameters.  A larger
+ * list is rejected with TULA_ERR_SCRATCH_LIMIT before anything is enqueued.
  *
  * Set-up: the first call on each device, with that device current, looks up the array's device
  * address (cudaGetSymbolAddress); make that first call before any stream capture.
@@ -195,7 +195,7 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
  * and must not be issued.  Allocates nothing: no cudaMalloc, no cudaFree, no allocating library
  * call.  Arguments, semantics and other status codes are those of tula_ags_step.
  */
-#define TULA_STATIC_SCRATCH_BYTES (4u << 20)
+#define TULA_STATIC_SCRATCH_BYTES (16u << 20)
 int tula_ags_step_static_scratch(float *const *param_ptrs, float *const *grad_ptrs,
                                  float *const *mom_ptrs, const int64_t *numels, int n_tensors,
                                  float lr, float momentum, float weight_decay,

@@ -20,7 +20,7 @@ c_int, c_float, c_void_p, c_size_t = ctypes.c_int, ctypes.c_float, ctypes.c_void
 
 TULA_OK, TULA_ERR_ARG, TULA_ERR_WORKSPACE, TULA_ERR_CUDA, TULA_ERR_UNSUPPORTED = 0, -1, -2, -3, -4
 TULA_ERR_SCRATCH_LIMIT = -5
-TULA_STATIC_SCRATCH_BYTES = 4 << 20
+TULA_STATIC_SCRATCH_BYTES = 16 << 20
 TULA_MAX_K = 16
 TULA_RULE_AGS, TULA_RULE_NONE, TULA_RULE_LARS, TULA_RULE_STATIC = 0, 1, 2, 3
 TULA_SCALE_PER_TENSOR, TULA_SCALE_PER_ELEMENT = 0, 1
@@ -282,6 +282,9 @@ class AGSOptimizerStep:
         self._g = _tensor_ptrs(flat)
         self._m = _tensor_ptrs(self.moms) if self.moms is not None else None
         self._numels = _numels(self.params)
+        # The zero fills above ran on the current stream; steps may be issued on any other
+        # (torch's side streams do not wait for it), so finish them before the first step.
+        torch.cuda.synchronize(dev)
 
     def set_trace_events(self, events):
         """cudaEvent_t handles (or None) recorded before pass 1, between passes, after pass 2."""
