@@ -124,8 +124,7 @@ typedef struct tula_ags_hparams {
  * static_s 1, lars_trust 1; all pointers NULL, grid_ctas 0. */
 void tula_ags_default_hparams(tula_ags_hparams *hp, int K);
 
-/* Bytes of workspace needed for this list of tensor sizes (host only; K does not change it
- * today and is validated). */
+/* Bytes of workspace needed for this list of tensor sizes and K replicas (host only). */
 int tula_ags_workspace_size(const int64_t *numels, int n_tensors, int K, size_t *bytes);
 
 /*
@@ -211,14 +210,29 @@ int tula_ags_last_cuda_error(void);
 uint64_t tula_ags_launch_count(void);
 
 /*
- * Host-only view of the work decomposition: tensor p is split into
- * max(1, ceil(numels[p] / tula_ags_chunk_elems())) chunks; chunk_start_out[p] is the index of
- * its first chunk and chunk_start_out[n_tensors] the total (n_tensors + 1 entries).
+ * Elements per tile (work item) of a pass that streams `streams` tensors through shared memory
+ * (the reduction pass: K replicas [+ w] [+ g_small]; the update pass: gbar, w [+ m] [+ per-element
+ * scale]): one tile of every stream fills one 32 KB stage.  A multiple of 128; TULA_ERR_ARG when
+ * streams is outside [1, TULA_MAX_K + 2].
  */
-int tula_ags_plan_chunks(const int64_t *numels, int n_tensors, int64_t *chunk_start_out);
+int tula_ags_chunk_elems(int streams);
 
-/* Elements per chunk (work item) of the reduction and update passes. */
-int tula_ags_chunk_elems(void);
+/*
+ * Host-only view of the work decomposition: tensor p is split into
+ * max(1, ceil(numels[p] / chunk_elems)) tiles; chunk_start_out[p] is the index of its first tile
+ * and chunk_start_out[n_tensors] the total (n_tensors + 1 entries).
+ */
+int tula_ags_plan_chunks(const int64_t *numels, int n_tensors, int chunk_elems,
+                         int64_t *chunk_start_out);
+
+/*
+ * Reads (synchronously, with cudaMemcpy) and clears the workspace's error word: 0 when every
+ * wait of the kernels that used this workspace completed; bit 0 set when a bounded wait inside a
+ * kernel ran out (the step's results are then not valid).  numels, n_tensors and K are those the
+ * workspace was sized for.
+ */
+int tula_ags_workspace_error(const void *workspace, size_t workspace_bytes,
+                             const int64_t *numels, int n_tensors, int K, int *error_out);
 
 #ifdef __cplusplus
 }

@@ -1,31 +1,40 @@
 // libtula_ags: the AGS optimizer step (Tula, arXiv 2603.18112) for sm_103a.
 //
-// Two streaming passes over every parameter tensor, load-balanced by a chunk
-// table: each tensor is cut into chunks of kChunk elements (tiny tensors are one
-// chunk, 100M-element tensors tens of thousands) and every chunk is one warp's
-// work item, so the streaming loops contain no block-wide barrier:
+// Per step, three kernels on the caller's stream, chained by programmatic
+// dependent launch so that each one's launch and prologue overlap the tail of
+// the one before:
 //
-//   k_reduce  (pass 1)  K-way replica mean (Eq. 1c) written over replica 0, and
-//                       fp64 per-chunk partial sums of |gbar|^2, |g_0|^2 [, |w|^2].
-//                       Partials are combined in a fixed order in two levels
-//                       (32-chunk groups, then the tensor) by whichever warp takes
-//                       the last ticket of a group / of a tensor; that warp also
-//                       derives the tensor's statistics, its coefficient when
-//                       scaled (the old gradscale, Eq. 8's s, or the LARS ratio)
-//                       and, when asked, the refreshed gradscale (UpdateGradScale,
-//                       Algorithm 1).  The warp finishing the last tensor forms
-//                       |G|^2, Delta (Eq. 5) and the branch of Algorithm 1.
-//   k_update  (pass 2)  d = c gbar + wd w; m = mu m + d; w = w - lr m (Eq. 7b with
-//                       the wrapped SGD), in reverse chunk order so that it starts
-//                       on the mean lines pass 1 left in L2; |w|^2 for statistics.
+//   k_reduce   (pass 1)  K-way replica mean (Eq. 1c) written over replica 0, and
+//                        fp64 per-tile partial sums of |gbar|^2, |g_0|^2 [, |w|^2].
+//   k_combine            per tensor, the fixed-order sum of its tile partials,
+//                        its statistics, its coefficient when scaled (the old
+//                        gradscale, Eq. 8's s, or the LARS ratio) and, when
+//                        asked, the refreshed gradscale (UpdateGradScale,
+//                        Algorithm 1); the CTA finishing last forms |G|^2,
+//                        Delta (Eq. 5) and the branch of Algorithm 1.
+//   k_update   (pass 2)  d = c gbar + wd w; m = mu m + d; w = w - lr m (Eq. 7b with
+//                        the wrapped SGD); |w|^2 per tile for the statistics
+//                        (then a k_combine of those).
 //
-// No warp ever waits on another: hand-offs are counter tickets.  Both kernels
-// are HBM-bound (a few flops per 20-70 bytes): 128-bit coalesced loads, one
-// wave of resident CTAs, no tensor cores (nothing here is a contraction).  The
-// chunk table, pointers and sizes travel in the kernel parameter block
-// (__grid_constant__, up to ~31 KB per launch), so no host-to-device copy,
+// The streaming passes: each tensor is cut into tiles of T elements (T fixed
+// per pass by how many tensors it streams, so that one tile of every stream
+// fills a 32 KB shared-memory stage).  One persistent CTA per SM takes tiles
+// round-robin.  Its producer warp moves tiles from HBM into a 6-stage ring
+// with TMA bulk copies (cp.async.bulk ... mbarrier::complete_tx), one copy per
+// stream issued by one lane each, so up to 192 KB per SM are in flight; three
+// consumer warps, each owning two stages, compute from shared memory and
+// release the stage through an mbarrier.  Consumers keep fp64 partial sums
+// per lane and reduce four tiles' worth at a time across the warp in a fixed
+// tree, so the FP64 latency chains overlap.  Only plain stores leave a tile.
+//
+// Every mbarrier wait is bounded; a wait that runs out sets an error word in
+// the workspace (tula_ags_workspace_error) and the CTA drains its copies in
+// flight and returns.  The streaming kernels are HBM-bound (a few flops per
+// 20-70 bytes); nothing here is a contraction, so no tensor cores.  The tile
+// table, pointers and sizes travel in the kernel parameter block
+// (__grid_constant__, up to ~31 KB per launch): no host-to-device copy,
 // allocation or host sync is ever needed.  The reduction order depends on the
-// numels only: results are bitwise reproducible and independent of the grid.
+// numels only, so results are bitwise reproducible and independent of the grid.
 #include "tula_ags.h"
 
 #include <cuda_runtime.h>
@@ -37,19 +46,31 @@
 #include <cstring>
 #include <memory>
 #include <mutex>
+#include <utility>
 #include <vector>
 
 namespace {
 
-constexpr int kThreads = 512;            // threads per CTA (16 independent warps)
-constexpr int kChunk = 4096;             // elements per chunk = one warp's work item
-constexpr int kGroup = 32;               // chunks per first-level combine group
-constexpr int kParamBudget = 31 * 1024;  // kernel parameter bytes per launch (limit 32764)
-constexpr int kAcc = 3;                  // partial sums per chunk: |gbar|^2, |g_0|^2, |w|^2
-constexpr int kTsum = 4;                 // per-tensor sums (stride)
+constexpr int kStageBytes = 32 * 1024;  // one tile of every stream
+constexpr int kStages = 6;              // ring depth (192 KB per CTA)
+constexpr int kConsumers = 3;           // consumer warps; consumer c owns stages c and c + 3
+constexpr int kThreads = 32 * (1 + kConsumers);
+constexpr int kSmemBytes = kStages * kStageBytes + 2 * kStages * 8;
+constexpr int kPend = 4;                // tiles whose warp reductions run together
+constexpr int kCombWarps = 4;           // k_combine: one warp per segment, 4 per CTA
+constexpr int kSegTiles = 256;          // tile partials per combine segment (8 per lane)
+constexpr int kParamBudget = 31 * 1024; // kernel parameter bytes per launch (limit 32764)
+constexpr int kAcc = 3;                 // partial sums per pass-1 tile: |gbar|^2, |g_0|^2, |w|^2
+constexpr int kTsum = 4;                // per-tensor sums (stride)
 constexpr unsigned kFull = 0xffffffffu;
+constexpr uint32_t kSpinLimit = 1u << 22;  // bound on every mbarrier wait (>= 1 s)
 
-enum Mode { kModeStep = 0, kModeStats = 1, kModeScale = 2 };
+enum Mode { kModeStep = 0, kModeStats = 1, kModeScale = 2, kModeUpdate = 3 };
+
+// Elements per tile when `streams` tensors share one 32 KB stage (multiple of 128).
+__host__ __device__ constexpr int tile_elems(int streams) {
+    return (kStageBytes / (4 * streams)) / 128 * 128;
+}
 
 // ----------------------------------------------------------------------------
 // Launch tables (kernel parameters)
@@ -57,17 +78,31 @@ enum Mode { kModeStep = 0, kModeStats = 1, kModeScale = 2 };
 
 template <int NP>
 struct Table {
-    static constexpr int kMaxT = (kParamBudget - 64) / (NP * 8 + 16);
-    int n;    // tensors in this launch
-    int t0;   // global index of its first tensor
-    int c0;   // global index of its first chunk
-    int nc;   // chunks in this launch
-    int g0;   // global index of its first combine group
+    static constexpr int kMaxT = (kParamBudget - 64) / (NP * 8 + 12);
+    int n;      // tensors in this launch
+    int t0;     // global index of its first tensor
+    int c0;     // global index of its first tile
+    int nc;     // tiles in this launch
+    int chunk;  // elements per tile
     int pad[3];
     long long numel[kMaxT];
-    int cstart[kMaxT + 1];  // first chunk of each tensor, relative to c0; cstart[n] = nc
-    int gstart[kMaxT + 1];  // first group of each tensor, relative to g0
+    int cstart[kMaxT + 1];  // first tile of each tensor, relative to c0; cstart[n] = nc
     const float *ptr[kMaxT][NP];
+};
+
+// k_combine: where each tensor's tile partials are, cut into segments of at
+// most kSegTiles tiles.
+struct CombTable {
+    static constexpr int kMaxT = 1536;
+    static constexpr int kMaxS = (kParamBudget - 64 - 12 * (kMaxT + 1)) / 2;
+    int n;   // tensors in this launch
+    int t0;  // global index of its first tensor
+    int s0;  // global index of its first segment
+    int ns;  // segments in this launch
+    int cfirst[kMaxT];          // global index of the tensor's first tile
+    int ntiles[kMaxT];          // its tile count
+    int sfirst[kMaxT + 1];      // its first segment, relative to s0; sfirst[n] = ns
+    unsigned short seg_t[kMaxS];  // the tensor (index in this launch) of each segment
 };
 
 struct Scalars {
@@ -77,28 +112,36 @@ struct Scalars {
     float *scale;
     double *state;
     double *stats;
-    unsigned *gctr1, *gctr2;  // per-group chunk tickets, pass 1 / pass 2
-    unsigned *tctr1, *tctr2;  // per-tensor group tickets, pass 1 / pass 2
-    unsigned *done;           // [0]: tensors finished in pass 1
-    int *flags;               // [0]: branch of the last step (1 = scaled)
-    double *partials;         // [chunk][kAcc]
-    double *gpart;            // [group][kAcc]
-    double *tsum;             // [tensor][kTsum]: |gbar|^2, |g_0|^2, |w|^2
-    float *cand;              // [tensor]: c_p of the scaled branch (AGS: the old gradscale)
+    unsigned *done;  // [0]: tensors combined after pass 1
+    int *flags;      // [0]: branch of the last step (1 = scaled)
+    unsigned *err;   // [0]: bounded waits that ran out (sticky until read)
+    unsigned *sctr1; // [tensor]: segments combined, pass 1
+    unsigned *sctr2; // [tensor]: segments combined, pass 2
+    double *part1;   // [tile][kAcc], pass 1
+    double *part2;   // [tile], pass 2 (|w|^2)
+    double *spart1;  // [segment][kAcc], pass 1
+    double *spart2;  // [segment], pass 2
+    double *tsum;    // [tensor][kTsum]: |gbar|^2, |g_0|^2, |w|^2
+    float *cand;     // [tensor]: c_p of the scaled branch (AGS: the old gradscale)
 };
 
 // ----------------------------------------------------------------------------
-// Device helpers
+// Device helpers: memory, arithmetic
 // ----------------------------------------------------------------------------
 
-__device__ __forceinline__ float4 ld_stream(const float *p) {
-    return __ldcs(reinterpret_cast<const float4 *>(p));
-}
 __device__ __forceinline__ void st_stream(float *p, float4 v) {
     __stcs(reinterpret_cast<float4 *>(p), v);
 }
 __device__ __forceinline__ void st_keep(float *p, float4 v) {
     *reinterpret_cast<float4 *>(p) = v;
+}
+// 16-byte load from shared memory (a shared-window address).
+__device__ __forceinline__ float4 lds4(uint32_t addr) {
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(addr));
+    return v;
 }
 
 // fp32 sum of squares into a running fp32 partial, one FFMA per term
@@ -125,25 +168,118 @@ __device__ __forceinline__ float4 add4(float4 a, float4 b) {
 }
 
 // Eq. 1c: divide the k-ascending sum by K (exact reciprocal when K is a power of 2)
+template <int KT>
 __device__ __forceinline__ float mean1(float s, const Scalars &sc) {
-    return sc.pow2K ? __fmul_rn(s, sc.invK) : __fdiv_rn(s, sc.Kf);
+    if constexpr (KT > 0 && (KT & (KT - 1)) == 0) {
+        return __fmul_rn(s, 1.0f / (float)KT);
+    } else if constexpr (KT > 0) {
+        return __fdiv_rn(s, (float)KT);
+    } else {
+        return sc.pow2K ? __fmul_rn(s, sc.invK) : __fdiv_rn(s, sc.Kf);
+    }
 }
+template <int KT>
 __device__ __forceinline__ float4 mean4(float4 s, const Scalars &sc) {
-    return make_float4(mean1(s.x, sc), mean1(s.y, sc), mean1(s.z, sc), mean1(s.w, sc));
+    return make_float4(mean1<KT>(s.x, sc), mean1<KT>(s.y, sc), mean1<KT>(s.z, sc),
+                       mean1<KT>(s.w, sc));
 }
 
-// Warp sum in a fixed tree (lane 0's result), broadcast to every lane.
-__device__ __forceinline__ double warp_sum(double v) {
+
+// Fixed-tree warp sum of R values at once (lane 0 gets the sums); the R chains
+// are independent, so their shuffle and fp64 add latencies overlap.
+template <int R>
+__device__ __forceinline__ void warp_sums(double (&v)[R]) {
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v = __dadd_rn(v, __shfl_down_sync(kFull, v, o));
-    return __shfl_sync(kFull, v, 0);
+    for (int o = 16; o > 0; o >>= 1) {
+        double t[R];
+#pragma unroll
+        for (int r = 0; r < R; ++r) t[r] = __shfl_down_sync(kFull, v[r], o);
+#pragma unroll
+        for (int r = 0; r < R; ++r) v[r] = __dadd_rn(v[r], t[r]);
+    }
 }
 
-// UpdateGradScale on tensor norms: min(|g_s| / (|g_l| + eps), s_max), fp64, rounded once.
-__device__ __forceinline__ float scale_tensor(double s_small, double s_large, const Scalars &sc) {
-    double q = sqrt(s_small) / (sqrt(s_large) + (double)sc.eps);
-    return (float)fmin(q, (double)sc.s_max);
+template <int R>
+__device__ __forceinline__ void warp_sums(float (&v)[R]) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        float t[R];
+#pragma unroll
+        for (int r = 0; r < R; ++r) t[r] = __shfl_down_sync(kFull, v[r], o);
+#pragma unroll
+        for (int r = 0; r < R; ++r) v[r] = __fadd_rn(v[r], t[r]);
+    }
 }
+
+// ----------------------------------------------------------------------------
+// Device helpers: programmatic dependent launch, mbarrier, TMA (inline PTX)
+// ----------------------------------------------------------------------------
+
+// Wait for the grids this one depends on to complete and their memory to be
+// visible, then let the next grid in the stream begin launching.
+__device__ __forceinline__ void grid_dependency() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_fence_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive_tx(uint64_t *bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+                 "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(uint64_t *bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Waits for the phase of `bar` with this parity to complete; gives up after
+// kSpinLimit tries (returns false).  try_wait suspends the thread in hardware
+// until the phase completes or a short time limit passes; only a wait that is
+// already far too long backs off with a sleep.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity) {
+    for (uint32_t i = 0; i < kSpinLimit; ++i) {
+        if (mbar_test(bar, parity)) return true;
+        if (i >= (1u << 16)) __nanosleep(256);
+    }
+    return false;
+}
+// One TMA bulk copy global -> shared, completing `bytes` of `bar`'s transaction count.
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t bytes,
+                                         uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+            "r"(dst),
+        "l"(src), "r"(bytes), "r"(smem_addr(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void report_timeout(const Scalars &sc) {
+    atomicOr(sc.err, 1u);
+}
+
+// ----------------------------------------------------------------------------
+// Tile table lookups
+// ----------------------------------------------------------------------------
 
 __device__ __forceinline__ int find_tensor(const int *cstart, int n, int c) {
     int lo = 0, hi = n;  // cstart[lo] <= c < cstart[hi]
@@ -154,142 +290,449 @@ __device__ __forceinline__ int find_tensor(const int *cstart, int n, int c) {
     return lo;
 }
 
-// Where a chunk sits: its tensor, its range and the global indices of its
-// tensor's first chunk and first group.
-struct ChunkPos {
-    int t, tg, c_in_t, nch, ngr;
-    long long begin, end, cfirst, gfirst;
+// Follows the tensor index along a monotone sequence of tiles (one CTA's tiles,
+// ascending or descending): O(1) per tile instead of a search.
+struct Walker {
+    int t = -1;
+    template <int NP>
+    __device__ __forceinline__ int to(const Table<NP> &tab, int c) {
+        if (t < 0) return t = find_tensor(tab.cstart, tab.n, c);
+        while (c >= tab.cstart[t + 1]) ++t;
+        while (c < tab.cstart[t]) --t;
+        return t;
+    }
+};
+
+// A tile: its tensor, its element range.
+struct TilePos {
+    int t, tg, c_in_t;
+    long long begin, end;
 };
 
 template <int NP>
-__device__ __forceinline__ ChunkPos locate(const Table<NP> &tab, int c) {
-    ChunkPos q;
-    q.t = find_tensor(tab.cstart, tab.n, c);
-    q.tg = tab.t0 + q.t;
-    q.c_in_t = c - tab.cstart[q.t];
-    q.nch = tab.cstart[q.t + 1] - tab.cstart[q.t];
-    q.ngr = tab.gstart[q.t + 1] - tab.gstart[q.t];
-    q.begin = (long long)q.c_in_t * kChunk;
-    q.end = min(q.begin + (long long)kChunk, tab.numel[q.t]);
-    q.cfirst = (long long)tab.c0 + tab.cstart[q.t];
-    q.gfirst = (long long)tab.g0 + tab.gstart[q.t];
+__device__ __forceinline__ TilePos locate(const Table<NP> &tab, int c, int t, int chunk) {
+    TilePos q;
+    q.t = t;
+    q.tg = tab.t0 + t;
+    q.c_in_t = c - tab.cstart[t];
+    q.begin = (long long)q.c_in_t * chunk;
+    q.end = min(q.begin + (long long)chunk, tab.numel[t]);
     return q;
 }
 
-// Hand-off of one chunk's partial sums (every lane holds acc[]).  Lane 0 stores
-// them and takes a ticket of the chunk's 32-chunk group; the warp holding the
-// group's last ticket adds the group's partials (lane i <- chunk i, then a
-// fixed tree) and takes a ticket of the tensor; the warp holding the tensor's
-// last ticket adds the group sums (lane-strided in order, then a fixed tree).
-// Returns true, with the tensor's sums in tot[] (every lane), on that warp only.
-// Counters are re-armed to zero by the warp that took their last ticket.
-template <int NA>
-__device__ __forceinline__ bool hand_off(const double (&acc)[NA], int slot, const ChunkPos &q,
-                                         double *partials, double *gpart, unsigned *gctr,
-                                         unsigned *tctr, double (&tot)[NA]) {
+// Float4 a tile moves by TMA: its 16-byte body when every stream of the tensor
+// is 16-byte aligned (lane i < ns holds stream i's pointer), else none.
+__device__ __forceinline__ int tile_vecs(const float *mine, int ns, const TilePos &q) {
+    if (q.end <= q.begin) return 0;
+    const unsigned low = (threadIdx.x & 31) < ns ? (unsigned)(reinterpret_cast<uintptr_t>(mine) & 15u)
+                                                 : 0u;
+    return __reduce_or_sync(kFull, low) == 0u ? (int)((q.end - q.begin) >> 2) : 0;
+}
+
+// The tensor of the previous tile, kept while the next tile stays in it: its
+// index, its streams' alignment and the lane's stream pointer, so a tile in
+// the same tensor needs no table look-up.
+struct TensorCache {
+    Walker walk;
+    int t = -1;
+    long long numel = 0;
+    const float *mine = nullptr;
+    bool aligned = false;
+    int nv = 0;  // float4 moved by TMA for the last tile asked for
+    template <int NP>
+    __device__ __forceinline__ TilePos at(const Table<NP> &tab, int c, int chunk, int role, int ns) {
+        const int tn = walk.to(tab, c);
+        if (tn != t) {
+            t = tn;
+            numel = tab.numel[t];
+            mine = (threadIdx.x & 31) < ns ? tab.ptr[t][role] : nullptr;
+            const unsigned low =
+                (threadIdx.x & 31) < ns ? (unsigned)(reinterpret_cast<uintptr_t>(mine) & 15u) : 0u;
+            aligned = __reduce_or_sync(kFull, low) == 0u;
+        }
+        TilePos q;
+        q.t = t;
+        q.tg = tab.t0 + t;
+        q.c_in_t = c - tab.cstart[t];
+        q.begin = (long long)q.c_in_t * chunk;
+        q.end = min(q.begin + (long long)chunk, numel);
+        nv = (aligned && q.end > q.begin) ? (int)((q.end - q.begin) >> 2) : 0;
+        return q;
+    }
+};
+
+// ----------------------------------------------------------------------------
+// The producer: TMA bulk copies of each tile's streams into the stage ring
+// ----------------------------------------------------------------------------
+//
+// Tile j of this CTA (launch tile blockIdx.x + j * gridDim.x, or its mirror
+// image when `reverse`) goes to stage j % kStages and is consumed by consumer
+// warp j % kConsumers.  The whole producer warp works on a tile: lane i < ns
+// fetches stream i's pointer (role roles[i]) and issues that stream's copy, to
+// offset i * chunk floats of the stage, after lane 0 has posted the tile's
+// byte count on the stage's full barrier.
+
+template <int NP, int NS>
+__device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
+                                        const int (&roles)[NS], int ns, int chunk, int ntiles,
+                                        bool reverse, uint32_t ring, uint64_t *full,
+                                        uint64_t *empty) {
     const int lane = threadIdx.x & 31;
-    const int grp = q.c_in_t / kGroup;
-    const int gsize = min(kGroup, q.nch - grp * kGroup);
-    const long long cg = q.cfirst + q.c_in_t;
-    const long long gg = q.gfirst + grp;
-    int last = 0;
+    const int role = lane < ns ? roles[lane] : 0;
+    TensorCache tc;
+    int issued = 0;
+    for (int j = 0; j < ntiles; ++j) {
+        const int s = j % kStages;
+        if (j >= kStages) {
+            int ok = 1;
+            if (lane == 0) ok = mbar_wait(&empty[s], (uint32_t)((j / kStages - 1) & 1));
+            if (!__shfl_sync(kFull, ok, 0)) {
+                if (lane == 0) report_timeout(sc);
+                break;
+            }
+        }
+        const int i = blockIdx.x + j * gridDim.x;
+        const int c = reverse ? tab.nc - 1 - i : i;
+        const TilePos q = tc.at(tab, c, chunk, role, ns);
+        const uint32_t bytes = 16u * (uint32_t)tc.nv;
+        if (lane == 0) mbar_arrive_tx(&full[s], bytes * (uint32_t)ns);
+        __syncwarp();
+        if (bytes && lane < ns)
+            bulk_g2s(ring + (uint32_t)s * kStageBytes + (uint32_t)(lane * chunk * 4),
+                     tc.mine + q.begin, bytes, &full[s]);
+        issued = j + 1;
+    }
+    // Drain: never leave the CTA with a copy still writing into its shared memory.
     if (lane == 0) {
-#pragma unroll
-        for (int a = 0; a < NA; ++a) partials[cg * kAcc + slot + a] = acc[a];
-        __threadfence();
-        last = atomicAdd(&gctr[gg], 1u) == (unsigned)(gsize - 1);
+        for (int s = 0; s < kStages && s < issued; ++s) {
+            const int jl = s + ((issued - 1 - s) / kStages) * kStages;  // last tile on stage s
+            if (!mbar_wait(&full[s], (uint32_t)((jl / kStages) & 1))) report_timeout(sc);
+        }
     }
-    if (!__shfl_sync(kFull, last, 0)) return false;
-    __threadfence();
-    double g[NA];
-    const long long c0 = q.cfirst + (long long)grp * kGroup;
-#pragma unroll
-    for (int a = 0; a < NA; ++a) {
-        g[a] = lane < gsize ? __ldcg(&partials[(c0 + lane) * kAcc + slot + a]) : 0.0;
-        g[a] = warp_sum(g[a]);
+}
+
+// Shared prologue of the streaming kernels: barrier init, tile count.
+__device__ __forceinline__ int ring_setup(unsigned char *smem, uint64_t *&full, uint64_t *&empty,
+                                          int nc) {
+    full = reinterpret_cast<uint64_t *>(smem + kStages * kStageBytes);
+    empty = full + kStages;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
+        mbar_fence_init();
     }
-    if (q.ngr == 1) {  // a single group is the whole tensor
-        if (lane == 0) gctr[gg] = 0u;
-#pragma unroll
-        for (int a = 0; a < NA; ++a) tot[a] = g[a];
-        return true;
-    }
-    last = 0;
-    if (lane == 0) {
-#pragma unroll
-        for (int a = 0; a < NA; ++a) gpart[gg * kAcc + slot + a] = g[a];
-        gctr[gg] = 0u;
-        __threadfence();
-        last = atomicAdd(&tctr[q.tg], 1u) == (unsigned)(q.ngr - 1);
-    }
-    if (!__shfl_sync(kFull, last, 0)) return false;
-    __threadfence();
-#pragma unroll
-    for (int a = 0; a < NA; ++a) tot[a] = 0.0;
-    for (int i = lane; i < q.ngr; i += 32) {
-#pragma unroll
-        for (int a = 0; a < NA; ++a)
-            tot[a] = __dadd_rn(tot[a], __ldcg(&gpart[(q.gfirst + i) * kAcc + slot + a]));
-    }
-#pragma unroll
-    for (int a = 0; a < NA; ++a) tot[a] = warp_sum(tot[a]);
-    if (lane == 0) tctr[q.tg] = 0u;
-    return true;
+    __syncthreads();
+    return (int)blockIdx.x < nc ? (nc - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x : 0;
 }
 
 // ----------------------------------------------------------------------------
-// Per-tensor results of pass 1 (lane 0 of the warp that finished the tensor)
+// Pass 1: replica mean + per-tile squared norms
 // ----------------------------------------------------------------------------
+//
+// Template: KT = replicas known at compile time (0: runtime K <= 16);
+// WM = write the mean over replica 0; RW = also reduce |w|^2;
+// SS = g_small is a separate stream instead of replica 0;
+// PR = precise norms: every exact fp64 square is added in fp64, and the tile's
+// lanes in an fp64 tree (relative error ~1e-15), for norms that feed a
+// per-tensor coefficient (UpdateGradScale, LARS).  Otherwise the tile's sum
+// stays in fp32: each lane adds <= 16 squares per group of 4 columns, then the
+// group sums, then a 5-level tree across lanes, a relative error below 71 ulp
+// (4e-6) of the tile's sum; tiles are combined in fp64.  That is what the
+// variability metric and the statistics need, and it keeps GB300's slow FP64
+// pipe out of the streaming loop.
+// Pointer roles per tensor: [0, K) replicas, KS = w, KS + 1 = g_small.
+// Stage streams: replicas 0..K-1, then w (RW), then g_small (SS).
 
-__device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, double sw) {
+template <int KT>
+struct P1 {
+    static constexpr int KS = KT > 0 ? KT : TULA_MAX_K;
+    static constexpr int NP = KS + 2;
+};
+
+// One float4 column of a tile: mean, squares.  x0 = replica 0, s = sum.
+template <int KT, bool WM, bool RW, bool SS, bool PR>
+__device__ __forceinline__ void column1(float4 x0, float4 s, float4 wv, float4 sv, float *out,
+                                        const Scalars &sc, int K, double &ag, double &as,
+                                        double &aw, float &pg, float &ps, float &pw) {
+    if (K > 1) {
+        s = mean4<KT>(s, sc);
+        if (WM) st_keep(out, s);
+    }
+    if (PR) {
+        ag = dsq4(ag, s);
+        if (K > 1) as = dsq4(as, x0);
+        if (SS) as = dsq4(as, sv);
+        if (RW) aw = dsq4(aw, wv);
+    } else {
+        pg = sq4(pg, s);
+        if (K > 1) ps = sq4(ps, x0);
+        if (SS) ps = sq4(ps, sv);
+        if (RW) pw = sq4(pw, wv);
+    }
+}
+
+// Per-lane partial sums of one tile (not yet reduced across the warp).
+template <int KT, bool WM, bool RW, bool SS, bool PR>
+__device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const float *const *ptr,
+                                            const TilePos &q, int nv, const Scalars &sc,
+                                            double (&accd)[kAcc], float (&accf)[kAcc]) {
+    constexpr int KS = P1<KT>::KS;
+    const int lane = threadIdx.x & 31;
+    const int K = KT > 0 ? KT : sc.K;
+    const uint32_t sw_s = stage + (uint32_t)(K * chunk * 4);
+    const uint32_t ss_s = stage + (uint32_t)((K + (RW ? 1 : 0)) * chunk * 4);
+    float *out = const_cast<float *>(ptr[0]) + q.begin;
+    double ag = 0.0, as = 0.0, aw = 0.0;  // precise (PR) sums
+    float fg = 0.f, fs = 0.f, fw = 0.f;   // fp32 sums (not PR)
+
+    if constexpr (KT > 0) {
+        constexpr int CH = tile_elems(KT + (RW ? 1 : 0) + (SS ? 1 : 0));
+        constexpr int COLS = CH / 128;  // float4 columns per lane of a full tile
+        if (nv == CH / 4) {
+            // Full tile: every lane has COLS columns; all loads of a column issue together.
+#pragma unroll
+            for (int c0 = 0; c0 < COLS; c0 += 4) {
+                float pg = 0.f, ps = 0.f, pw = 0.f;
+#pragma unroll
+                for (int u = 0; u < 4; ++u) {
+                    if (c0 + u < COLS) {
+                        const int v = lane + 32 * (c0 + u);
+                        float4 x[KT];
+#pragma unroll
+                        for (int k = 0; k < KT; ++k)
+                            x[k] = lds4(stage + (uint32_t)((k * CH + 4 * v) * 4));
+                        const float4 wv = RW ? lds4(sw_s + (uint32_t)(16 * v)) : x[0];
+                        const float4 sv = SS ? lds4(ss_s + (uint32_t)(16 * v)) : x[0];
+                        float4 s = x[0];
+#pragma unroll
+                        for (int k = 1; k < KT; ++k) s = add4(s, x[k]);
+                        column1<KT, WM, RW, SS, PR>(x[0], s, wv, sv, out + 4 * v, sc, K, ag, as,
+                                                    aw, pg, ps, pw);
+                    }
+                }
+                if (!PR) {
+                    fg = __fadd_rn(fg, pg);
+                    if (K > 1 || SS) fs = __fadd_rn(fs, ps);
+                    if (RW) fw = __fadd_rn(fw, pw);
+                }
+            }
+            nv = -1;  // done
+        }
+    }
+    if (nv >= 0) {
+        // Ragged tile, or K known only at run time.
+        for (int v0 = lane; v0 < nv; v0 += 32 * 4) {
+            float pg = 0.f, ps = 0.f, pw = 0.f;
+            for (int u = 0; u < 4; ++u) {
+                const int v = v0 + 32 * u;
+                if (v >= nv) break;
+                const float4 x0 = lds4(stage + (uint32_t)(16 * v));
+                float4 s = x0;
+                for (int k = 1; k < K; ++k)
+                    s = add4(s, lds4(stage + (uint32_t)((k * chunk + 4 * v) * 4)));
+                const float4 wv = RW ? lds4(sw_s + (uint32_t)(16 * v)) : x0;
+                const float4 sv = SS ? lds4(ss_s + (uint32_t)(16 * v)) : x0;
+                column1<KT, WM, RW, SS, PR>(x0, s, wv, sv, out + 4 * v, sc, K, ag, as, aw, pg, ps,
+                                            pw);
+            }
+            if (!PR) {
+                fg = __fadd_rn(fg, pg);
+                if (K > 1 || SS) fs = __fadd_rn(fs, ps);
+                if (RW) fw = __fadd_rn(fw, pw);
+            }
+        }
+        // Tail (< 4 elements) or a misaligned tensor: plain loads from global memory.
+        for (long long j = q.begin + 4 * (long long)nv + lane; j < q.end; j += 32) {
+            const float x0 = __ldcs(ptr[0] + j);
+            float s = x0;
+            for (int k = 1; k < K; ++k) s = __fadd_rn(s, __ldcs(ptr[k] + j));
+            if (K > 1) {
+                s = mean1<KT>(s, sc);
+                if (WM) const_cast<float *>(ptr[0])[j] = s;
+            }
+            const float y_s = SS ? __ldcs(ptr[KS + 1] + j) : 0.f;
+            const float y_w = RW ? __ldcs(ptr[KS] + j) : 0.f;
+            if (PR) {
+                if (K > 1) as = __fma_rn((double)x0, (double)x0, as);
+                ag = __fma_rn((double)s, (double)s, ag);
+                if (SS) as = __fma_rn((double)y_s, (double)y_s, as);
+                if (RW) aw = __fma_rn((double)y_w, (double)y_w, aw);
+            } else {
+                if (K > 1) fs = __fmaf_rn(x0, x0, fs);
+                fg = __fmaf_rn(s, s, fg);
+                if (SS) fs = __fmaf_rn(y_s, y_s, fs);
+                if (RW) fw = __fmaf_rn(y_w, y_w, fw);
+            }
+        }
+    }
+    if (PR) {
+        accd[0] = ag;
+        accd[1] = (K > 1 || SS) ? as : ag;  // K = 1: replica 0 is the mean
+        accd[2] = aw;
+    } else {
+        accf[0] = fg;
+        accf[1] = (K > 1 || SS) ? fs : fg;
+        accf[2] = fw;
+    }
+}
+
+template <int KT, bool WM, bool RW, bool SS, bool PR>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_reduce(const __grid_constant__ Table<P1<KT>::NP> tab, const __grid_constant__ Scalars sc) {
+    constexpr int KS = P1<KT>::KS;
+    constexpr int NSMAX = KS + 2;
+    extern __shared__ __align__(128) unsigned char smem[];
+    grid_dependency();
+    uint64_t *full, *empty;
+    const int ntiles = ring_setup(smem, full, empty, tab.nc);
+    const uint32_t ring = smem_addr(smem);
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int K = KT > 0 ? KT : sc.K;
+    const int chunk = tab.chunk;
+    int roles[NSMAX];
+    int ns = 0;
+    for (int k = 0; k < K; ++k) roles[ns++] = k;
+    if (RW) roles[ns++] = KS;
+    if (SS) roles[ns++] = KS + 1;
+    if (warp == 0) {
+        produce<P1<KT>::NP, NSMAX>(tab, sc, roles, ns, chunk, ntiles, false, ring, full, empty);
+        return;
+    }
+    const int my_role = lane < ns ? roles[lane] : 0;
+
+    const int cw = warp - 1;
+    TensorCache tc;
+    for (int jb = cw; jb < ntiles; jb += kConsumers * kPend) {
+        double pendd[PR ? kPend * kAcc : 1];
+        float pendf[PR ? 1 : kPend * kAcc];
+        int ptile[kPend];
+        bool stop = false;
+#pragma unroll
+        for (int p = 0; p < kPend; ++p) {
+            const int j = jb + p * kConsumers;
+            ptile[p] = -1;
+#pragma unroll
+            for (int a = 0; a < kAcc; ++a) {
+                if constexpr (PR) pendd[p * kAcc + a] = 0.0;
+                else pendf[p * kAcc + a] = 0.f;
+            }
+            if (stop || j >= ntiles) continue;
+            const int s = j % kStages;
+            const int c = blockIdx.x + j * gridDim.x;
+            const TilePos q = tc.at(tab, c, chunk, my_role, ns);
+            const float *const *ptr = tab.ptr[q.t];
+            if (!mbar_wait(&full[s], (uint32_t)((j / kStages) & 1))) {
+                if (lane == 0) report_timeout(sc);
+                stop = true;
+                continue;
+            }
+            double accd[kAcc];
+            float accf[kAcc];
+            reduce_tile<KT, WM, RW, SS, PR>(ring + (uint32_t)s * kStageBytes, chunk, ptr, q,
+                                            tc.nv, sc, accd, accf);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[s]);
+            ptile[p] = tab.c0 + c;
+#pragma unroll
+            for (int a = 0; a < kAcc; ++a) {
+                if constexpr (PR) pendd[p * kAcc + a] = accd[a];
+                else pendf[p * kAcc + a] = accf[a];
+            }
+        }
+        if constexpr (PR) warp_sums<kPend * kAcc>(pendd);
+        else warp_sums<kPend * kAcc>(pendf);
+        if (lane == 0) {
+#pragma unroll
+            for (int p = 0; p < kPend; ++p)
+                if (ptile[p] >= 0) {
+                    double *P = sc.part1 + (size_t)ptile[p] * kAcc;
+#pragma unroll
+                    for (int a = 0; a < kAcc; ++a) {
+                        if constexpr (PR) P[a] = pendd[p * kAcc + a];
+                        else P[a] = (double)pendf[p * kAcc + a];
+                    }
+                }
+        }
+        if (stop) break;
+    }
+}
+
+// ----------------------------------------------------------------------------
+// k_combine: per-tensor fixed-order sums of the tile partials
+// ----------------------------------------------------------------------------
+//
+// One warp per segment of at most kSegTiles tile partials of one tensor (no
+// block barrier; GB300's FP64 pipe sees 15 warp-wide adds per segment).  A
+// tensor of several segments is finished by the warp taking its last segment
+// ticket.  After pass 1 (NA = kAcc) the sums give the tensor's statistics and
+// coefficients; in step mode each tensor then takes a ticket and the warp
+// taking the last one forms |G|^2, Delta and the branch.  After pass 2
+// (NA = 1) the sum is |w|^2 for the statistics.
+
+// Per-tensor results after pass 1, by the whole warp that finished the tensor
+// (its sums in lane 0).  The square roots of |gbar|^2, |g_0|^2 and |w|^2 are
+// taken by lanes 0, 1, 2 in one instruction.
+__device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, double sw,
+                            float old) {
+    const int lane = threadIdx.x & 31;
+    sg = __shfl_sync(kFull, sg, 0);
+    ss = __shfl_sync(kFull, ss, 0);
+    sw = __shfl_sync(kFull, sw, 0);
+    const double r = sqrt(lane == 0 ? sg : (lane == 1 ? ss : sw));
+    const double ng = __shfl_sync(kFull, r, 0), ns = __shfl_sync(kFull, r, 1),
+                 nw = __shfl_sync(kFull, r, 2);
+    if (lane != 0) return;
     double *T = sc.tsum + (size_t)tg * kTsum;
     T[0] = sg;
     T[1] = ss;
     T[2] = sw;
     double *row = sc.stats ? sc.stats + (size_t)tg * TULA_STATS_LEN : nullptr;
     if (sc.mode == kModeScale) {
-        sc.scale[tg] = scale_tensor(ss, sg, sc);  // g_0 = g_large, small = g_small
+        // UpdateGradScale, g_0 = g_large, small = g_small: min(|g_s| / (|g_l| + eps), s_max)
+        sc.scale[tg] = (float)fmin(ns / (ng + (double)sc.eps), (double)sc.s_max);
         return;
     }
     if (sc.mode == kModeStats) {
         row[TULA_STAT_W_SQ] = sw;
         row[TULA_STAT_G_SQ] = sg;
         row[TULA_STAT_G0_SQ] = ss;
-        row[TULA_STAT_W_NORM] = sqrt(sw);
-        row[TULA_STAT_G_NORM] = sqrt(sg);
-        row[TULA_STAT_RATIO] = sg > 0.0 ? sqrt(sw) / sqrt(sg) : 0.0;
+        row[TULA_STAT_W_NORM] = nw;
+        row[TULA_STAT_G_NORM] = ng;
+        row[TULA_STAT_RATIO] = sg > 0.0 ? nw / ng : 0.0;
         row[TULA_STAT_COEF] = 0.0;
         row[TULA_STAT_SCALE] = 0.0;
         return;
     }
     // kModeStep: the coefficient this tensor gets when the step is scaled (Algorithm 1,
     // Eq. 8) or always (LARS), before UpdateGradScale may overwrite gradscale.
-    const float old = sc.scale ? sc.scale[tg] : 1.0f;
     float cand;
     switch (sc.rule) {
     case TULA_RULE_AGS: cand = old; break;
     case TULA_RULE_STATIC: cand = sc.static_s; break;
     case TULA_RULE_LARS:
-        cand = (sw > 0.0 && sg > 0.0) ? (float)((double)sc.lars_trust * (sqrt(sw) / sqrt(sg)))
-                                      : 1.0f;
+        cand = (sw > 0.0 && sg > 0.0) ? (float)((double)sc.lars_trust * (nw / ng)) : 1.0f;
         break;
     default: cand = 1.0f;
     }
     sc.cand[tg] = cand;
     float s_after = sc.scale ? old : 0.0f;
     if (sc.refresh && sc.scale) {
-        s_after = scale_tensor(ss, sg, sc);
+        // UpdateGradScale with g_small = replica 0 and g_large = the mean
+        s_after = (float)fmin(ns / (ng + (double)sc.eps), (double)sc.s_max);
         sc.scale[tg] = s_after;
     }
     if (row) {
         row[TULA_STAT_G_SQ] = sg;
         row[TULA_STAT_G0_SQ] = ss;
-        row[TULA_STAT_G_NORM] = sqrt(sg);
+        row[TULA_STAT_G_NORM] = ng;
         row[TULA_STAT_SCALE] = (double)s_after;
         if (sc.read_w) {
             row[TULA_STAT_W_SQ] = sw;
-            row[TULA_STAT_W_NORM] = sqrt(sw);
-            row[TULA_STAT_RATIO] = sg > 0.0 ? sqrt(sw) / sqrt(sg) : 0.0;
+            row[TULA_STAT_W_NORM] = nw;
+            row[TULA_STAT_RATIO] = sg > 0.0 ? nw / ng : 0.0;
         }
     }
 }
@@ -298,11 +741,12 @@ __device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, dou
 // tensor's sums are in sc.tsum).
 __device__ void finalize_step(const Scalars &sc) {
     const int lane = threadIdx.x & 31;
-    double v = 0.0;
+    double v[1] = {0.0};
     for (int t = lane; t < sc.n_total; t += 32)
-        v = __dadd_rn(v, __ldcg(&sc.tsum[(size_t)t * kTsum + 0]));
-    const double g2 = warp_sum(v);
+        v[0] = __dadd_rn(v[0], __ldcg(&sc.tsum[(size_t)t * kTsum + 0]));
+    warp_sums<1>(v);
     if (lane != 0) return;
+    const double g2 = v[0];
     const double g2_prev = sc.state[TULA_STATE_G2_PREV];
     const double steps = sc.state[TULA_STATE_STEPS];
     // no previous step -> +inf (sensitive)
@@ -319,196 +763,96 @@ __device__ void finalize_step(const Scalars &sc) {
     sc.done[0] = 0u;  // re-arm for the next call
 }
 
-// ----------------------------------------------------------------------------
-// Pass 1: replica mean + per-tensor squared norms
-// ----------------------------------------------------------------------------
-//
-// Template: KT = replicas known at compile time (0: runtime K <= 16);
-// WM = write the mean over replica 0; RW = also reduce |w|^2;
-// SS = g_small is a separate stream (role KS + 1) instead of replica 0;
-// PR = precise norms: every exact fp64 square is added in fp64 (relative error
-// ~1e-15), for norms that feed a per-tensor coefficient (UpdateGradScale, LARS);
-// otherwise each lane sums <= 16 squares in fp32 before one fp64 add (~1e-7),
-// which is what the variability metric and the statistics need, at a fraction
-// of GB300's FP64 rate.
-// Pointer roles per tensor: [0, K) replicas, KS = w, KS + 1 = g_small.
-
-template <int KT>
-struct P1 {
-    static constexpr int KS = KT > 0 ? KT : TULA_MAX_K;
-    static constexpr int NP = KS + 2;
-};
-
-template <int KT, bool WM, bool RW, bool SS, bool PR>
-__device__ __forceinline__ void reduce_vec(const float *const *ptr, long long begin, int nv,
-                                           const Scalars &sc, double &ag, double &as,
-                                           double &aw) {
-    constexpr int KS = P1<KT>::KS;
-    constexpr int NS = (KT > 0 ? KT : 4) + (RW ? 1 : 0) + (SS ? 1 : 0);  // streams read
-    constexpr int U = NS >= 4 ? 1 : 4 / NS;  // >= 4 float4 loads per lane in flight
-    constexpr int KL = KT > 0 ? KT : TULA_MAX_K;  // load slots
+template <int NA>
+__global__ void __launch_bounds__(32 * kCombWarps)
+    k_combine(const __grid_constant__ CombTable tab, const __grid_constant__ Scalars sc) {
+    grid_dependency();
     const int lane = threadIdx.x & 31;
-    const int K = KT > 0 ? KT : sc.K;
-    const float *g[KL];
-#pragma unroll
-    for (int k = 0; k < KL; ++k) g[k] = (KT > 0 && k < K) ? ptr[k] + begin : nullptr;
-    const float *wp = RW ? ptr[KS] + begin : nullptr;
-    const float *sp = SS ? ptr[KS + 1] + begin : nullptr;
-    float *out = const_cast<float *>(ptr[0]) + begin;
+    const int seg = (int)blockIdx.x * kCombWarps + (int)(threadIdx.x >> 5);
+    if (seg >= tab.ns) return;
+    const int t = tab.seg_t[seg];
+    const int tg = tab.t0 + t;
+    // gradscale of this tensor, needed by the epilogue: load it now (AGS step)
+    const float scale_old = (NA == kAcc && sc.mode == kModeStep && sc.scale) ? sc.scale[tg] : 1.0f;
+    const int k = seg - tab.sfirst[t];                 // segment within the tensor
+    const int nseg = tab.sfirst[t + 1] - tab.sfirst[t];
+    const double *part = NA == kAcc ? sc.part1 : sc.part2;
+    double *spart = NA == kAcc ? sc.spart1 : sc.spart2;
+    unsigned *sctr = NA == kAcc ? sc.sctr1 : sc.sctr2;
+    const long long first = (long long)tab.cfirst[t] + (long long)k * kSegTiles;
+    const int n = min(kSegTiles, tab.ntiles[t] - k * kSegTiles);
 
-    if constexpr (KT == 0) {
-        // K not known at compile time: replicas 1..K-1 in groups of four, k ascending.
-#pragma unroll 1
-        for (int v = lane; v < nv; v += 32) {
-            const float4 x0 = ld_stream(ptr[0] + begin + 4 * (size_t)v);
-            float4 s = x0;
-            for (int k0 = 1; k0 < K; k0 += 4) {
-                float4 y[4];
+    // The segment's tiles: lane i adds tiles i, i + 32, ... in order (8 loads in
+    // flight), then a fixed tree across the warp.
+    double v[NA];
 #pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    if (k0 + j < K) y[j] = ld_stream(ptr[k0 + j] + begin + 4 * (size_t)v);
+    for (int a = 0; a < NA; ++a) v[a] = 0.0;
+    int i = lane;
+    for (; i + 7 * 32 < n; i += 8 * 32) {
+        double x[8][NA];
 #pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    if (k0 + j < K) s = add4(s, y[j]);
-            }
-            s = mean4(s, sc);
-            if (WM) st_keep(out + 4 * (size_t)v, s);
-            float4 wv = RW ? ld_stream(wp + 4 * (size_t)v) : s;
-            float4 sv = SS ? ld_stream(sp + 4 * (size_t)v) : s;
-            if (PR) {
-                as = dsq4(as, x0);
-                ag = dsq4(ag, s);
-                if (SS) as = dsq4(as, sv);
-                if (RW) aw = dsq4(aw, wv);
-            } else {
-                as = __dadd_rn(as, (double)sq4(0.f, x0));
-                ag = __dadd_rn(ag, (double)sq4(0.f, s));
-                if (SS) as = __dadd_rn(as, (double)sq4(0.f, sv));
-                if (RW) aw = __dadd_rn(aw, (double)sq4(0.f, wv));
-            }
-        }
-        return;
+        for (int u = 0; u < 8; ++u)
+#pragma unroll
+            for (int a = 0; a < NA; ++a) x[u][a] = part[(first + i + 32 * u) * NA + a];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+#pragma unroll
+            for (int a = 0; a < NA; ++a) v[a] = __dadd_rn(v[a], x[u][a]);
     }
-
-#pragma unroll 1
-    for (int v0 = lane; v0 < nv; v0 += 32 * U) {
-        float4 x[U][KL];
-        float4 wv[U], sv[U];
+    for (; i < n; i += 32) {
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int v = v0 + u * 32;
-            if (v < nv) {
-#pragma unroll
-                for (int k = 0; k < KL; ++k)
-                    if (k < K) x[u][k] = ld_stream(g[k] + 4 * (size_t)v);
-                if (RW) wv[u] = ld_stream(wp + 4 * (size_t)v);
-                if (SS) sv[u] = ld_stream(sp + 4 * (size_t)v);
-            }
-        }
-        float pg = 0.f, ps = 0.f, pw = 0.f;
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int v = v0 + u * 32;
-            if (v < nv) {
-                float4 s = x[u][0];
-#pragma unroll
-                for (int k = 1; k < KL; ++k)
-                    if (k < K) s = add4(s, x[u][k]);
-                if (K > 1) {
-                    s = mean4(s, sc);
-                    if (WM) st_keep(out + 4 * (size_t)v, s);
-                    if (PR) as = dsq4(as, x[u][0]); else ps = sq4(ps, x[u][0]);
-                }
-                if (PR) {
-                    ag = dsq4(ag, s);
-                    if (SS) as = dsq4(as, sv[u]);
-                    if (RW) aw = dsq4(aw, wv[u]);
-                } else {
-                    pg = sq4(pg, s);
-                    if (SS) ps = sq4(ps, sv[u]);
-                    if (RW) pw = sq4(pw, wv[u]);
-                }
-            }
-        }
-        if (!PR) {
-            ag = __dadd_rn(ag, (double)pg);
-            if (K > 1 || SS) as = __dadd_rn(as, (double)ps);
-            if (RW) aw = __dadd_rn(aw, (double)pw);
-        }
+        for (int a = 0; a < NA; ++a) v[a] = __dadd_rn(v[a], part[(first + i) * NA + a]);
     }
-}
+    warp_sums<NA>(v);
 
-template <int KT, bool WM, bool RW, bool SS>
-__device__ __forceinline__ void reduce_scalar(const float *const *ptr, long long j0, long long j1,
-                                              const Scalars &sc, double &ag, double &as,
-                                              double &aw) {
-    constexpr int KS = P1<KT>::KS;
-    constexpr int KL = KT > 0 ? KT : TULA_MAX_K;
-    const int K = KT > 0 ? KT : sc.K;
-    for (long long j = j0 + (threadIdx.x & 31); j < j1; j += 32) {
-        float x0 = __ldcs(ptr[0] + j);
-        float s = x0;
-#pragma unroll
-        for (int k = 1; k < KL; ++k)
-            if (k < K) s = __fadd_rn(s, __ldcs(ptr[k] + j));
-        if (K > 1) {
-            s = mean1(s, sc);
-            if (WM) const_cast<float *>(ptr[0])[j] = s;
-            as = __fma_rn((double)x0, (double)x0, as);
-        }
-        ag = __fma_rn((double)s, (double)s, ag);
-        if (SS) {
-            const double y = __ldcs(ptr[KS + 1] + j);
-            as = __fma_rn(y, y, as);
-        }
-        if (RW) {
-            const double y = __ldcs(ptr[KS] + j);
-            aw = __fma_rn(y, y, aw);
-        }
-    }
-}
-
-template <int KT, bool WM, bool RW, bool SS, bool PR>
-__global__ void __launch_bounds__(kThreads, 2)
-    k_reduce(const __grid_constant__ Table<P1<KT>::NP> tab, const __grid_constant__ Scalars sc) {
-    constexpr int KS = P1<KT>::KS;
-    const int K = KT > 0 ? KT : sc.K;
-    const int warp = (int)((blockIdx.x * (unsigned)kThreads + threadIdx.x) >> 5);
-    const int nwarps = (int)((gridDim.x * (unsigned)kThreads) >> 5);
-
-    for (int c = warp; c < tab.nc; c += nwarps) {
-        const ChunkPos q = locate(tab, c);
-        const float *const *ptr = tab.ptr[q.t];
-        double acc[kAcc] = {0.0, 0.0, 0.0};
-        if (q.end > q.begin) {
-            uintptr_t al = 0;
-            for (int k = 0; k < K; ++k) al |= reinterpret_cast<uintptr_t>(ptr[k]);
-            if (RW) al |= reinterpret_cast<uintptr_t>(ptr[KS]);
-            if (SS) al |= reinterpret_cast<uintptr_t>(ptr[KS + 1]);
-            const int nv = (al & 15u) == 0 ? (int)((q.end - q.begin) >> 2) : 0;
-            if (nv > 0)
-                reduce_vec<KT, WM, RW, SS, PR>(ptr, q.begin, nv, sc, acc[0], acc[1], acc[2]);
-            reduce_scalar<KT, WM, RW, SS>(ptr, q.begin + 4 * (long long)nv, q.end, sc, acc[0],
-                                          acc[1], acc[2]);
-        }
-#pragma unroll
-        for (int a = 0; a < kAcc; ++a) acc[a] = warp_sum(acc[a]);
-        double tot[kAcc];
-        if (!hand_off<kAcc>(acc, 0, q, sc.partials, sc.gpart, sc.gctr1, sc.tctr1, tot)) continue;
-        // This warp finished tensor q.tg.
-        if ((threadIdx.x & 31) == 0) {
-            const double ss = (K > 1 || SS) ? tot[1] : tot[0];  // K = 1: replica 0 is the mean
-            tensor_done(sc, q.tg, tot[0], ss, tot[2]);
-        }
-        if (sc.mode != kModeStep) continue;
+    if (nseg > 1) {
+        // Hand the segment sum over; the warp taking the tensor's last ticket adds
+        // the segment sums in order.
         int last = 0;
-        if ((threadIdx.x & 31) == 0) {
+        const long long sg0 = (long long)tab.s0 + tab.sfirst[t];
+        if (lane == 0) {
+#pragma unroll
+            for (int a = 0; a < NA; ++a) spart[(sg0 + k) * NA + a] = v[a];
             __threadfence();
-            last = atomicAdd(&sc.done[0], 1u) == (unsigned)(sc.n_total - 1);
+            last = atomicAdd(&sctr[tg], 1u) == (unsigned)(nseg - 1);
+        }
+        if (!__shfl_sync(kFull, last, 0)) return;
+        __threadfence();
+#pragma unroll
+        for (int a = 0; a < NA; ++a) v[a] = 0.0;
+        for (int j = lane; j < nseg; j += 32) {
+#pragma unroll
+            for (int a = 0; a < NA; ++a) v[a] = __dadd_rn(v[a], __ldcg(&spart[(sg0 + j) * NA + a]));
+        }
+        warp_sums<NA>(v);
+        if (lane == 0) sctr[tg] = 0u;  // re-arm
+    }
+
+    // This warp holds tensor tg's sums (lane 0).
+    if constexpr (NA == kAcc) {
+        int last = 0;
+        tensor_done(sc, tg, v[0], v[1], v[2], scale_old);
+        if (lane == 0) {
+            if (sc.mode == kModeStep) {
+                __threadfence();
+                last = atomicAdd(&sc.done[0], 1u) == (unsigned)(sc.n_total - 1);
+            }
         }
         if (__shfl_sync(kFull, last, 0)) {
             __threadfence();
             finalize_step(sc);
+        }
+    } else {
+        // lanes 0 and 1 take the two square roots in one instruction
+        const double sw = __shfl_sync(kFull, v[0], 0);
+        const double sg = sc.tsum[(size_t)tg * kTsum + 0];
+        const double r = sqrt(lane == 0 ? sw : sg);
+        const double nw = __shfl_sync(kFull, r, 0), ng = __shfl_sync(kFull, r, 1);
+        if (lane == 0) {
+            double *row = sc.stats + (size_t)tg * TULA_STATS_LEN;
+            row[TULA_STAT_W_SQ] = sw;
+            row[TULA_STAT_W_NORM] = nw;
+            row[TULA_STAT_RATIO] = sg > 0.0 ? nw / ng : 0.0;
         }
     }
 }
@@ -517,7 +861,8 @@ __global__ void __launch_bounds__(kThreads, 2)
 // Pass 2: scaled momentum-SGD + weight-decay update (Eq. 7b, Algorithm 1)
 // ----------------------------------------------------------------------------
 // Pointer roles: 0 = gbar, 1 = w, 2 = m, 3 = per-element gradscale.
-// Chunks run in reverse order: the mean pass 1 wrote last is still in L2.
+// Stage streams: gbar, w, then m (HM), then the per-element scale (PE, scaled).
+// Tiles run in reverse order: the mean pass 1 wrote last is still in L2.
 
 constexpr int kNP2 = 4;
 
@@ -533,99 +878,145 @@ __device__ __forceinline__ void sgd1(float g, float c, float &w, float &m, const
     }
 }
 
+// One float4 column of the update; returns the squares of w (before the update).
+template <bool HM>
+__device__ __forceinline__ float update4(float4 g4, float4 w4, float4 m4, float4 cc, float *wp,
+                                         float *mp, const Scalars &sc, float pw) {
+    pw = sq4(pw, w4);
+    sgd1(g4.x, cc.x, w4.x, m4.x, sc, HM);
+    sgd1(g4.y, cc.y, w4.y, m4.y, sc, HM);
+    sgd1(g4.z, cc.z, w4.z, m4.z, sc, HM);
+    sgd1(g4.w, cc.w, w4.w, m4.w, sc, HM);
+    st_stream(wp, w4);
+    if (HM) st_stream(mp, m4);
+    return pw;
+}
+
 template <bool HM, bool PE, bool SW>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, 1)
     k_update(const __grid_constant__ Table<kNP2> tab, const __grid_constant__ Scalars sc) {
-    constexpr int U = 2;
+    extern __shared__ __align__(128) unsigned char smem[];
+    grid_dependency();
+    uint64_t *full, *empty;
+    const int ntiles = ring_setup(smem, full, empty, tab.nc);
+    const uint32_t ring = smem_addr(smem);
+    const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int warp = (int)((blockIdx.x * (unsigned)kThreads + threadIdx.x) >> 5);
-    const int nwarps = (int)((gridDim.x * (unsigned)kThreads) >> 5);
+    const int chunk = tab.chunk;
     const int scaled = sc.flags[0];
     const bool gated = sc.rule == TULA_RULE_AGS || sc.rule == TULA_RULE_STATIC;
     const bool use_se = PE && scaled;
+    const int ns = 2 + (HM ? 1 : 0) + (use_se ? 1 : 0);
+    int roles[4] = {0, 1, 2, 3};
+    if (!HM) roles[2] = 3;
+    if (warp == 0) {
+        produce<kNP2, 4>(tab, sc, roles, ns, chunk, ntiles, true, ring, full, empty);
+        return;
+    }
+    const int my_role = lane < ns ? roles[lane] : 0;
+    constexpr int CH = tile_elems(2 + (HM ? 1 : 0) + (PE ? 1 : 0));
+    constexpr int COLS = CH / 128;
+    const uint32_t w_off = (uint32_t)(CH * 4);
+    const uint32_t m_off = (uint32_t)(2 * CH * 4);
+    const uint32_t se_off = (uint32_t)((HM ? 3 : 2) * CH * 4);
 
-    for (int i = warp; i < tab.nc; i += nwarps) {
-        const int c = tab.nc - 1 - i;
-        const ChunkPos q = locate(tab, c);
-        const float cand = sc.cand[q.tg];
-        const float ct = gated ? (scaled ? cand : 1.0f) : cand;
-        if (sc.stats && q.c_in_t == 0 && lane == 0)
-            sc.stats[(size_t)q.tg * TULA_STATS_LEN + TULA_STAT_COEF] =
-                PE ? (scaled ? (double)NAN : 1.0) : (double)ct;
-        double aw[1] = {0.0};
-
-        if (q.end > q.begin) {
+    TensorCache tc;
+    const int cw = warp - 1;
+    for (int jb = cw; jb < ntiles; jb += kConsumers * kPend) {
+        float pend[kPend];
+        int ptile[kPend];
+        bool stop = false;
+#pragma unroll
+        for (int p = 0; p < kPend; ++p) {
+            const int j = jb + p * kConsumers;
+            ptile[p] = -1;
+            pend[p] = 0.f;
+            if (stop || j >= ntiles) continue;
+            const int s = j % kStages;
+            const int c = tab.nc - 1 - ((int)blockIdx.x + j * (int)gridDim.x);
+            const TilePos q = tc.at(tab, c, chunk, my_role, ns);
             const float *const *ptr = tab.ptr[q.t];
-            const float *gp = ptr[0] + q.begin;
+            const int nv = tc.nv;
+            const float cand = sc.cand[q.tg];
+            const float ct = gated ? (scaled ? cand : 1.0f) : cand;
+            if (sc.stats && q.c_in_t == 0 && lane == 0)
+                sc.stats[(size_t)q.tg * TULA_STATS_LEN + TULA_STAT_COEF] =
+                    PE ? (scaled ? (double)NAN : 1.0) : (double)ct;
+            if (!mbar_wait(&full[s], (uint32_t)((j / kStages) & 1))) {
+                if (lane == 0) report_timeout(sc);
+                stop = true;
+                continue;
+            }
+            const uint32_t stage = ring + (uint32_t)s * kStageBytes;
             float *wp = const_cast<float *>(ptr[1]) + q.begin;
             float *mp = HM ? const_cast<float *>(ptr[2]) + q.begin : nullptr;
-            const float *sp = use_se ? ptr[3] + q.begin : nullptr;
-            uintptr_t al = reinterpret_cast<uintptr_t>(gp) | reinterpret_cast<uintptr_t>(wp);
-            if (HM) al |= reinterpret_cast<uintptr_t>(mp);
-            if (use_se) al |= reinterpret_cast<uintptr_t>(sp);
-            const int nv = (al & 15u) == 0 ? (int)((q.end - q.begin) >> 2) : 0;
-#pragma unroll 1
-            for (int v0 = lane; v0 < nv; v0 += 32 * U) {
-                float4 gv[U], wv[U], mv[U], sv[U];
+            const float4 cdef = PE ? make_float4(1.f, 1.f, 1.f, 1.f) : make_float4(ct, ct, ct, ct);
+            float aw = 0.f;  // fp32 |w|^2 of the tile (statistics only)
+            if (nv == CH / 4) {
 #pragma unroll
-                for (int u = 0; u < U; ++u) {
-                    const int v = v0 + u * 32;
-                    if (v < nv) {
-                        gv[u] = ld_stream(gp + 4 * (size_t)v);
-                        wv[u] = ld_stream(wp + 4 * (size_t)v);
-                        if (HM) mv[u] = ld_stream(mp + 4 * (size_t)v);
-                        if (use_se) sv[u] = ld_stream(sp + 4 * (size_t)v);
-                    }
-                }
-                float pw = 0.f;
+                for (int c0 = 0; c0 < COLS; c0 += 4) {
+                    float pw = 0.f;
 #pragma unroll
-                for (int u = 0; u < U; ++u) {
-                    const int v = v0 + u * 32;
-                    if (v < nv) {
-                        if (SW) pw = sq4(pw, wv[u]);
-                        float4 cc = use_se ? sv[u] : make_float4(ct, ct, ct, ct);
-                        if (PE && !scaled) cc = make_float4(1.f, 1.f, 1.f, 1.f);
-                        float4 w4 = wv[u], m4 = HM ? mv[u] : make_float4(0.f, 0.f, 0.f, 0.f);
-                        sgd1(gv[u].x, cc.x, w4.x, m4.x, sc, HM);
-                        sgd1(gv[u].y, cc.y, w4.y, m4.y, sc, HM);
-                        sgd1(gv[u].z, cc.z, w4.z, m4.z, sc, HM);
-                        sgd1(gv[u].w, cc.w, w4.w, m4.w, sc, HM);
-                        st_stream(wp + 4 * (size_t)v, w4);
-                        if (HM) st_stream(mp + 4 * (size_t)v, m4);
+                    for (int u = 0; u < 4; ++u) {
+                        if (c0 + u < COLS) {
+                            const int v = lane + 32 * (c0 + u);
+                            const float4 g4 = lds4(stage + (uint32_t)(16 * v));
+                            const float4 w4 = lds4(stage + w_off + (uint32_t)(16 * v));
+                            const float4 m4 = HM ? lds4(stage + m_off + (uint32_t)(16 * v)) : g4;
+                            const float4 cc =
+                                use_se ? lds4(stage + se_off + (uint32_t)(16 * v)) : cdef;
+                            pw = update4<HM>(g4, w4, m4, cc, wp + 4 * v, mp + 4 * v, sc, pw);
+                        }
                     }
+                    if (SW) aw = __fadd_rn(aw, pw);
                 }
-                if (SW) aw[0] = __dadd_rn(aw[0], (double)pw);
+            } else {
+                for (int v0 = lane; v0 < nv; v0 += 32 * 4) {
+                    float pw = 0.f;
+                    for (int u = 0; u < 4; ++u) {
+                        const int v = v0 + 32 * u;
+                        if (v >= nv) break;
+                        const float4 g4 = lds4(stage + (uint32_t)(16 * v));
+                        const float4 w4 = lds4(stage + w_off + (uint32_t)(16 * v));
+                        const float4 m4 = HM ? lds4(stage + m_off + (uint32_t)(16 * v)) : g4;
+                        const float4 cc = use_se ? lds4(stage + se_off + (uint32_t)(16 * v)) : cdef;
+                        pw = update4<HM>(g4, w4, m4, cc, wp + 4 * v, mp + 4 * v, sc, pw);
+                    }
+                    if (SW) aw = __fadd_rn(aw, pw);
+                }
             }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[s]);
             const long long n = q.end - q.begin;
-            for (long long j = 4 * (long long)nv + lane; j < n; j += 32) {
-                const float g = __ldcs(gp + j);
-                float w = __ldcs(wp + j);
-                float m = HM ? __ldcs(mp + j) : 0.f;
-                float cj = use_se ? __ldcs(sp + j) : (PE ? 1.f : ct);
-                if (SW) aw[0] = __fma_rn((double)w, (double)w, aw[0]);
+            for (long long jj = 4 * (long long)nv + lane; jj < n; jj += 32) {
+                const float g = __ldcs(ptr[0] + q.begin + jj);
+                float w = wp[jj];
+                float m = HM ? mp[jj] : 0.f;
+                const float cj = use_se ? __ldcs(ptr[3] + q.begin + jj) : (PE ? 1.f : ct);
+                if (SW) aw = __fmaf_rn(w, w, aw);
                 sgd1(g, cj, w, m, sc, HM);
-                __stcs(wp + j, w);
-                if (HM) __stcs(mp + j, m);
+                wp[jj] = w;
+                if (HM) mp[jj] = m;
+            }
+            ptile[p] = tab.c0 + c;
+            pend[p] = aw;
+        }
+        if (SW) {
+            warp_sums<kPend>(pend);
+            if (lane == 0) {
+#pragma unroll
+                for (int p = 0; p < kPend; ++p)
+                    if (ptile[p] >= 0) sc.part2[ptile[p]] = (double)pend[p];
             }
         }
-        if (!SW) continue;
-        aw[0] = warp_sum(aw[0]);
-        double tot[1];
-        if (!hand_off<1>(aw, 2, q, sc.partials, sc.gpart, sc.gctr2, sc.tctr2, tot)) continue;
-        if (lane == 0) {
-            const double sw = tot[0];
-            const double sg = __ldcg(&sc.tsum[(size_t)q.tg * kTsum + 0]);
-            double *row = sc.stats + (size_t)q.tg * TULA_STATS_LEN;
-            row[TULA_STAT_W_SQ] = sw;
-            row[TULA_STAT_W_NORM] = sqrt(sw);
-            row[TULA_STAT_RATIO] = sg > 0.0 ? sqrt(sw) / sqrt(sg) : 0.0;
-        }
+        if (stop) break;
     }
 }
 
 // ----------------------------------------------------------------------------
 // UpdateGradScale, element-wise (Algorithm 1): s = fminf(|gs / (gl + eps)|, s_max)
 // ----------------------------------------------------------------------------
+// A once-per-epoch call: plain 128-bit loads, one warp per tile.
 // Pointer roles: 0 = g_small, 1 = g_large, 2 = s_out.
 
 constexpr int kNP3 = 3;
@@ -634,25 +1025,25 @@ __device__ __forceinline__ float scale1(float gs, float gl, const Scalars &sc) {
     return fminf(fabsf(__fdiv_rn(gs, __fadd_rn(gl, sc.eps))), sc.s_max);
 }
 
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads)
     k_scale_elem(const __grid_constant__ Table<kNP3> tab, const __grid_constant__ Scalars sc) {
+    grid_dependency();
     const int lane = threadIdx.x & 31;
     const int warp = (int)((blockIdx.x * (unsigned)kThreads + threadIdx.x) >> 5);
     const int nwarps = (int)((gridDim.x * (unsigned)kThreads) >> 5);
+    Walker walk;
     for (int c = warp; c < tab.nc; c += nwarps) {
-        const ChunkPos q = locate(tab, c);
-        if (q.end <= q.begin) continue;
+        const TilePos q = locate(tab, c, walk.to(tab, c), tab.chunk);
         const float *const *ptr = tab.ptr[q.t];
+        const int nv = tile_vecs(lane < 3 ? ptr[lane] : nullptr, 3, q);
         const float *a = ptr[0] + q.begin;
         const float *b = ptr[1] + q.begin;
         float *o = const_cast<float *>(ptr[2]) + q.begin;
-        const uintptr_t al = reinterpret_cast<uintptr_t>(a) | reinterpret_cast<uintptr_t>(b) |
-                             reinterpret_cast<uintptr_t>(o);
-        const int nv = (al & 15u) == 0 ? (int)((q.end - q.begin) >> 2) : 0;
         for (int v = lane; v < nv; v += 32) {
-            const float4 x = ld_stream(a + 4 * (size_t)v), y = ld_stream(b + 4 * (size_t)v);
-            st_stream(o + 4 * (size_t)v, make_float4(scale1(x.x, y.x, sc), scale1(x.y, y.y, sc),
-                                                     scale1(x.z, y.z, sc), scale1(x.w, y.w, sc)));
+            const float4 x = __ldcs(reinterpret_cast<const float4 *>(a) + v);
+            const float4 y = __ldcs(reinterpret_cast<const float4 *>(b) + v);
+            st_stream(o + 4 * v, make_float4(scale1(x.x, y.x, sc), scale1(x.y, y.y, sc),
+                                             scale1(x.z, y.z, sc), scale1(x.w, y.w, sc)));
         }
         const long long n = q.end - q.begin;
         for (long long j = 4 * (long long)nv + lane; j < n; j += 32)
@@ -667,17 +1058,28 @@ __global__ void __launch_bounds__(kThreads, 2)
 std::atomic<uint64_t> g_launches{0};
 thread_local int g_last_cuda = 0;
 
-inline long long chunks_of(int64_t n) { return n <= 0 ? 1 : (n + kChunk - 1) / kChunk; }
-inline long long groups_of(long long nch) { return (nch + kGroup - 1) / kGroup; }
+inline long long tiles_of(int64_t n, int chunk) { return n <= 0 ? 1 : (n + chunk - 1) / chunk; }
+
+inline int replica_slot(int K) {
+    return (K == 1 || K == 2 || K == 4 || K == 8 || K == 16) ? K : TULA_MAX_K;
+}
+
+// Tile sizes: the smallest a pass can use for K replicas sizes the workspace.
+inline int chunk1(int K, bool rw, bool ss) { return tile_elems(K + (rw ? 1 : 0) + (ss ? 1 : 0)); }
+inline int chunk2(bool hm, bool pe) { return tile_elems(2 + (hm ? 1 : 0) + (pe ? 1 : 0)); }
+inline int chunk1_min(int K) { return chunk1(K, true, K == 1); }
+inline int chunk2_min() { return chunk2(true, true); }
+
+inline long long segs_of(long long tiles) { return (tiles + kSegTiles - 1) / kSegTiles; }
 
 struct Plan {
-    long long chunks = 0, groups = 0;
+    long long c1 = 0, c2 = 0, s1 = 0, s2 = 0;  // tiles and combine segments of each pass
 };
 
-// Workspace layout.  Every counter and flag precedes `partials`, so zeroing
-// [0, partials) clears all of them.
+// Workspace layout.  Every counter and flag precedes `part1`, so zeroing
+// [0, part1) clears all of them.
 struct WsLayout {
-    size_t gctr1, gctr2, tctr1, tctr2, done, flags, partials, gpart, tsum, cand, total;
+    size_t done, flags, err, sctr1, sctr2, part1, part2, spart1, spart2, tsum, cand, total;
 };
 
 WsLayout ws_layout(int n_tensors, const Plan &pl) {
@@ -688,29 +1090,33 @@ WsLayout ws_layout(int n_tensors, const Plan &pl) {
         return o;
     };
     WsLayout L;
-    L.gctr1 = take(sizeof(unsigned) * (size_t)pl.groups);
-    L.gctr2 = take(sizeof(unsigned) * (size_t)pl.groups);
-    L.tctr1 = take(sizeof(unsigned) * (size_t)n_tensors);
-    L.tctr2 = take(sizeof(unsigned) * (size_t)n_tensors);
     L.done = take(sizeof(unsigned) * 4);
     L.flags = take(sizeof(int) * 4);
-    L.partials = take(sizeof(double) * kAcc * (size_t)pl.chunks);
-    L.gpart = take(sizeof(double) * kAcc * (size_t)pl.groups);
+    L.err = take(sizeof(unsigned) * 4);
+    L.sctr1 = take(sizeof(unsigned) * (size_t)n_tensors);
+    L.sctr2 = take(sizeof(unsigned) * (size_t)n_tensors);
+    L.part1 = take(sizeof(double) * kAcc * (size_t)pl.c1);
+    L.part2 = take(sizeof(double) * (size_t)pl.c2);
+    L.spart1 = take(sizeof(double) * kAcc * (size_t)pl.s1);
+    L.spart2 = take(sizeof(double) * (size_t)pl.s2);
     L.tsum = take(sizeof(double) * kTsum * (size_t)n_tensors);
     L.cand = take(sizeof(float) * (size_t)n_tensors);
     L.total = off;
     return L;
 }
 
-bool valid_numels(const int64_t *numels, int n, Plan *pl) {
-    if (!numels || n < 1) return false;
+bool valid_numels(const int64_t *numels, int n, int K, Plan *pl) {
+    if (!numels || n < 1 || K < 1 || K > TULA_MAX_K) return false;
+    const int t1 = chunk1_min(K), t2 = chunk2_min();
     Plan p;
     for (int i = 0; i < n; ++i) {
         if (numels[i] < 0) return false;
-        const long long c = chunks_of(numels[i]);
-        p.chunks += c;
-        p.groups += groups_of(c);
-        if (p.chunks >= (1LL << 31)) return false;
+        const long long a = tiles_of(numels[i], t1), b = tiles_of(numels[i], t2);
+        p.c1 += a;
+        p.c2 += b;
+        p.s1 += segs_of(a);
+        p.s2 += segs_of(b);
+        if (p.c1 >= (1LL << 31) || p.c2 >= (1LL << 31)) return false;
     }
     *pl = p;
     return true;
@@ -718,80 +1124,135 @@ bool valid_numels(const int64_t *numels, int n, Plan *pl) {
 
 inline bool aligned4(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 3u) == 0; }
 
-// One wave of resident CTAs for `kernel` on the current device (cached).
-int resident_ctas(const void *kernel) {
+// One wave of resident CTAs of `kernel` on the current device (cached); sets
+// the kernel's dynamic shared memory limit on first use.
+int resident_ctas(const void *kernel, int threads, int smem) {
     struct Entry { const void *k; int dev; int ctas; };
     static std::mutex mu;
     static std::vector<Entry> cache;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-    {
-        std::lock_guard<std::mutex> lock(mu);
-        for (const Entry &e : cache)
-            if (e.k == kernel && e.dev == dev) return e.ctas;
-    }
+    std::lock_guard<std::mutex> lock(mu);
+    for (const Entry &e : cache)
+        if (e.k == kernel && e.dev == dev) return e.ctas;
+    if (smem > 48 * 1024 &&
+        cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+            cudaSuccess)
+        return 0;
     int sms = 0, per = 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, kernel, kThreads, 0) != cudaSuccess)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per, kernel, threads, smem) != cudaSuccess)
         return 0;
     const int ctas = std::max(1, sms * std::max(per, 1));
-    std::lock_guard<std::mutex> lock(mu);
     cache.push_back({kernel, dev, ctas});
     return ctas;
 }
 
-// Splits tensors [0, n) into parameter blocks and launches `kernel` once per
-// block (in reverse block order when `reverse`).  fill(p, ptrs) writes tensor
-// p's pointers.
+// Launch with programmatic stream serialization: the kernel may begin while
+// the previous kernel in the stream finishes; its griddepcontrol.wait orders
+// every memory access after that kernel's completion.
+template <typename... KArgs, typename... Args>
+int launch_pdl(void (*kernel)(KArgs...), int grid, int threads, int smem, cudaStream_t s,
+               Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3((unsigned)threads);
+    cfg.dynamicSmemBytes = (size_t)smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    if (e == cudaSuccess) e = cudaGetLastError();
+    if (e != cudaSuccess) {
+        g_last_cuda = (int)e;
+        return TULA_ERR_CUDA;
+    }
+    return TULA_OK;
+}
+
+// Splits tensors [0, n) into parameter blocks of tiles of `chunk` elements and
+// launches `kernel` once per block (in reverse block order when `reverse`).
+// fill(p, ptrs) writes tensor p's pointers.
 template <int NP, typename Kernel, typename Fill>
-int launch_groups(Kernel kernel, int n, const int64_t *numels, const Scalars &sc, int grid_override,
-                  cudaStream_t stream, Fill fill, bool reverse = false) {
+int launch_streaming(Kernel kernel, int n, const int64_t *numels, int chunk, int smem,
+                     const Scalars &sc, int grid_override, cudaStream_t stream, Fill fill,
+                     bool reverse = false) {
     using T = Table<NP>;
-    int grid_cap = grid_override > 0 ? grid_override : resident_ctas((const void *)kernel);
+    const int grid_cap = resident_ctas((const void *)kernel, kThreads, smem);
     if (grid_cap <= 0) {
         g_last_cuda = (int)cudaGetLastError();
         return TULA_ERR_CUDA;
     }
     std::vector<std::unique_ptr<T>> tabs;
-    long long c_global = 0, g_global = 0;
+    long long c_global = 0;
     int p = 0;
     while (p < n) {
         std::unique_ptr<T> tab(new T);
         std::memset(tab.get(), 0, sizeof(T));
         tab->t0 = p;
         tab->c0 = (int)c_global;
-        tab->g0 = (int)g_global;
-        int cnt = 0, nc = 0, ng = 0;
+        tab->chunk = chunk;
+        int cnt = 0, nc = 0;
         while (p < n && cnt < T::kMaxT) {
             tab->numel[cnt] = numels[p];
             tab->cstart[cnt] = nc;
-            tab->gstart[cnt] = ng;
             fill(p, tab->ptr[cnt]);
-            const long long c = chunks_of(numels[p]);
-            nc += (int)c;
-            ng += (int)groups_of(c);
+            nc += (int)tiles_of(numels[p], chunk);
             ++cnt;
             ++p;
         }
         tab->n = cnt;
         tab->nc = nc;
         tab->cstart[cnt] = nc;
-        tab->gstart[cnt] = ng;
         c_global += nc;
-        g_global += ng;
         tabs.push_back(std::move(tab));
     }
     if (reverse) std::reverse(tabs.begin(), tabs.end());
     for (const auto &tab : tabs) {
-        const int need = (tab->nc + kThreads / 32 - 1) / (kThreads / 32);  // one warp per chunk
-        const int grid = std::max(1, std::min(need, grid_cap));
-        kernel<<<grid, kThreads, 0, stream>>>(*tab, sc);
-        g_launches.fetch_add(1, std::memory_order_relaxed);
-        cudaError_t e = cudaGetLastError();
-        if (e != cudaSuccess) {
-            g_last_cuda = (int)e;
-            return TULA_ERR_CUDA;
+        int grid = grid_override > 0 ? grid_override : grid_cap;
+        grid = std::max(1, std::min(grid, tab->nc));
+        const int rc = launch_pdl(kernel, grid, kThreads, smem, stream, *tab, sc);
+        if (rc) return rc;
+    }
+    return TULA_OK;
+}
+
+// k_combine over all tensors (tiles of `chunk` elements), NA sums per tile.
+template <int NA>
+int launch_combine(int n, const int64_t *numels, int chunk, const Scalars &sc, cudaStream_t s) {
+    std::unique_ptr<CombTable> tab(new CombTable);
+    long long c_global = 0, s_global = 0;
+    int p = 0;
+    while (p < n) {
+        std::memset(tab.get(), 0, sizeof(CombTable));
+        tab->t0 = p;
+        tab->s0 = (int)s_global;
+        int cnt = 0, ns = 0;
+        while (p < n && cnt < CombTable::kMaxT) {
+            const long long c = tiles_of(numels[p], chunk);
+            const int segs = (int)segs_of(c);
+            if (ns + segs > CombTable::kMaxS) break;  // next launch
+            tab->cfirst[cnt] = (int)c_global;
+            tab->ntiles[cnt] = (int)c;
+            tab->sfirst[cnt] = ns;
+            for (int k = 0; k < segs; ++k) tab->seg_t[ns + k] = (unsigned short)cnt;
+            ns += segs;
+            c_global += c;
+            ++cnt;
+            ++p;
         }
+        if (cnt == 0) return TULA_ERR_UNSUPPORTED;  // one tensor with more segments than a table
+        tab->n = cnt;
+        tab->ns = ns;
+        tab->sfirst[cnt] = ns;
+        s_global += ns;
+        const int grid = (ns + kCombWarps - 1) / kCombWarps;
+        const int rc = launch_pdl(k_combine<NA>, grid, 32 * kCombWarps, 0, s, *tab, sc);
+        if (rc) return rc;
     }
     return TULA_OK;
 }
@@ -821,36 +1282,41 @@ Scalars make_scalars(const tula_ags_hparams *hp, int K, int n, void *ws, const W
         sc.stats = hp->layer_stats;
     }
     char *b = static_cast<char *>(ws);
-    sc.gctr1 = reinterpret_cast<unsigned *>(b + L.gctr1);
-    sc.gctr2 = reinterpret_cast<unsigned *>(b + L.gctr2);
-    sc.tctr1 = reinterpret_cast<unsigned *>(b + L.tctr1);
-    sc.tctr2 = reinterpret_cast<unsigned *>(b + L.tctr2);
     sc.done = reinterpret_cast<unsigned *>(b + L.done);
     sc.flags = reinterpret_cast<int *>(b + L.flags);
-    sc.partials = reinterpret_cast<double *>(b + L.partials);
-    sc.gpart = reinterpret_cast<double *>(b + L.gpart);
+    sc.err = reinterpret_cast<unsigned *>(b + L.err);
+    sc.sctr1 = reinterpret_cast<unsigned *>(b + L.sctr1);
+    sc.sctr2 = reinterpret_cast<unsigned *>(b + L.sctr2);
+    sc.part1 = reinterpret_cast<double *>(b + L.part1);
+    sc.part2 = reinterpret_cast<double *>(b + L.part2);
+    sc.spart1 = reinterpret_cast<double *>(b + L.spart1);
+    sc.spart2 = reinterpret_cast<double *>(b + L.spart2);
     sc.tsum = reinterpret_cast<double *>(b + L.tsum);
     sc.cand = reinterpret_cast<float *>(b + L.cand);
     return sc;
 }
 
-// Pass-1 dispatch over the compile-time replica count.
+// Pass 1 (+ its combine) dispatched over the compile-time replica count.
 template <int KT, bool WM, bool RW, bool SS, bool PR, typename Fill>
-int run_reduce_k(int n, const int64_t *numels, const Scalars &sc, int grid, cudaStream_t s,
+int run_reduce_k(int K, int n, const int64_t *numels, const Scalars &sc, int grid, cudaStream_t s,
                  Fill fill) {
-    return launch_groups<P1<KT>::NP>(k_reduce<KT, WM, RW, SS, PR>, n, numels, sc, grid, s, fill);
+    const int chunk = chunk1(K, RW, SS);
+    int rc = launch_streaming<P1<KT>::NP>(k_reduce<KT, WM, RW, SS, PR>, n, numels, chunk,
+                                          kSmemBytes, sc, grid, s, fill);
+    if (rc) return rc;
+    return launch_combine<kAcc>(n, numels, chunk, sc, s);
 }
 
 template <bool WM, bool RW, bool SS, bool PR, typename Fill>
 int run_reduce(int K, int n, const int64_t *numels, const Scalars &sc, int grid, cudaStream_t s,
                Fill fill) {
     switch (K) {
-    case 1: return run_reduce_k<1, false, RW, SS, PR>(n, numels, sc, grid, s, fill);
-    case 2: return run_reduce_k<2, WM, RW, SS, PR>(n, numels, sc, grid, s, fill);
-    case 4: return run_reduce_k<4, WM, RW, SS, PR>(n, numels, sc, grid, s, fill);
-    case 8: return run_reduce_k<8, WM, RW, SS, PR>(n, numels, sc, grid, s, fill);
-    case 16: return run_reduce_k<16, WM, RW, SS, PR>(n, numels, sc, grid, s, fill);
-    default: return run_reduce_k<0, WM, RW, SS, PR>(n, numels, sc, grid, s, fill);
+    case 1: return run_reduce_k<1, false, RW, SS, PR>(K, n, numels, sc, grid, s, fill);
+    case 2: return run_reduce_k<2, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill);
+    case 4: return run_reduce_k<4, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill);
+    case 8: return run_reduce_k<8, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill);
+    case 16: return run_reduce_k<16, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill);
+    default: return run_reduce_k<0, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill);
     }
 }
 
@@ -863,10 +1329,6 @@ int check_ws(void *ws, size_t bytes, int n, const Plan &pl) {
 
 void record(void *ev, cudaStream_t s) {
     if (ev) cudaEventRecord(static_cast<cudaEvent_t>(ev), s);
-}
-
-inline int replica_slot(int K) {
-    return (K == 1 || K == 2 || K == 4 || K == 8 || K == 16) ? K : TULA_MAX_K;
 }
 
 }  // namespace
@@ -894,23 +1356,46 @@ void tula_ags_default_hparams(tula_ags_hparams *hp, int K) {
 
 int tula_ags_workspace_size(const int64_t *numels, int n_tensors, int K, size_t *bytes) {
     Plan pl;
-    if (!bytes || K < 1 || K > TULA_MAX_K || !valid_numels(numels, n_tensors, &pl))
-        return TULA_ERR_ARG;
+    if (!bytes || !valid_numels(numels, n_tensors, K, &pl)) return TULA_ERR_ARG;
     *bytes = ws_layout(n_tensors, pl).total;
     return TULA_OK;
 }
 
-int tula_ags_chunk_elems(void) { return kChunk; }
+int tula_ags_chunk_elems(int streams) {
+    if (streams < 1 || streams > TULA_MAX_K + 2) return TULA_ERR_ARG;
+    return tile_elems(streams);
+}
 
-int tula_ags_plan_chunks(const int64_t *numels, int n_tensors, int64_t *chunk_start_out) {
+int tula_ags_plan_chunks(const int64_t *numels, int n_tensors, int chunk_elems,
+                         int64_t *chunk_start_out) {
     Plan pl;
-    if (!chunk_start_out || !valid_numels(numels, n_tensors, &pl)) return TULA_ERR_ARG;
+    if (!chunk_start_out || chunk_elems < 1 || !valid_numels(numels, n_tensors, 1, &pl))
+        return TULA_ERR_ARG;
     int64_t c = 0;
     for (int p = 0; p < n_tensors; ++p) {
         chunk_start_out[p] = c;
-        c += chunks_of(numels[p]);
+        c += tiles_of(numels[p], chunk_elems);
     }
     chunk_start_out[n_tensors] = c;
+    return TULA_OK;
+}
+
+int tula_ags_workspace_error(const void *workspace, size_t workspace_bytes,
+                             const int64_t *numels, int n_tensors, int K, int *error_out) {
+    Plan pl;
+    if (!workspace || !error_out || !valid_numels(numels, n_tensors, K, &pl)) return TULA_ERR_ARG;
+    const WsLayout L = ws_layout(n_tensors, pl);
+    if (workspace_bytes < L.total) return TULA_ERR_WORKSPACE;
+    unsigned v = 0;
+    unsigned *dev = reinterpret_cast<unsigned *>(static_cast<char *>(const_cast<void *>(workspace)) +
+                                                 L.err);
+    cudaError_t e = cudaMemcpy(&v, dev, sizeof(v), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess && v) e = cudaMemset(dev, 0, sizeof(v));
+    if (e != cudaSuccess) {
+        g_last_cuda = (int)e;
+        return TULA_ERR_CUDA;
+    }
+    *error_out = (int)v;
     return TULA_OK;
 }
 
@@ -918,10 +1403,9 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
                   const int64_t *numels, int n_tensors, float lr, float momentum,
                   float weight_decay, const tula_ags_hparams *hp, void *stream) {
     Plan pl;
-    if (!hp || !param_ptrs || !grad_ptrs || !valid_numels(numels, n_tensors, &pl))
+    if (!hp || !param_ptrs || !grad_ptrs || !valid_numels(numels, n_tensors, hp->K, &pl))
         return TULA_ERR_ARG;
     const int K = hp->K, n = n_tensors;
-    if (K < 1 || K > TULA_MAX_K) return TULA_ERR_ARG;
     if (hp->rule < TULA_RULE_AGS || hp->rule > TULA_RULE_STATIC) return TULA_ERR_ARG;
     if (hp->granularity != TULA_SCALE_PER_TENSOR && hp->granularity != TULA_SCALE_PER_ELEMENT)
         return TULA_ERR_ARG;
@@ -983,8 +1467,11 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
     };
     const bool hm = mom_ptrs != nullptr;
     const bool sw = hp->layer_stats != nullptr && !lars;
-#define TULA_UPD(HM, PE, SW) \
-    launch_groups<kNP2>(k_update<HM, PE, SW>, n, numels, sc, hp->grid_ctas, s, fill2, true)
+    const int c2 = chunk2(hm, per_elem);
+    sc.mode = kModeUpdate;
+#define TULA_UPD(HM, PE, SW)                                                                       \
+    launch_streaming<kNP2>(k_update<HM, PE, SW>, n, numels, c2, kSmemBytes, sc, hp->grid_ctas, s, \
+                           fill2, true)
     if (hm) {
         if (per_elem) rc = sw ? TULA_UPD(true, true, true) : TULA_UPD(true, true, false);
         else rc = sw ? TULA_UPD(true, false, true) : TULA_UPD(true, false, false);
@@ -994,6 +1481,8 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
     }
 #undef TULA_UPD
     if (rc) return rc;
+    if (sw) rc = launch_combine<1>(n, numels, c2, sc, s);
+    if (rc) return rc;
     record(hp->trace_events[2], s);
     return TULA_OK;
 }
@@ -1002,9 +1491,8 @@ int tula_layer_stats(const float *const *param_ptrs, const float *const *grad_pt
                      const int64_t *numels, int n_tensors, double *stats_out, void *workspace,
                      size_t workspace_bytes, void *stream) {
     Plan pl;
-    if (!param_ptrs || !grad_ptrs || !stats_out || !valid_numels(numels, n_tensors, &pl))
+    if (!param_ptrs || !grad_ptrs || !stats_out || !valid_numels(numels, n_tensors, K, &pl))
         return TULA_ERR_ARG;
-    if (K < 1 || K > TULA_MAX_K) return TULA_ERR_ARG;
     const int n = n_tensors;
     for (int p = 0; p < n; ++p) {
         if (numels[p] == 0) continue;
@@ -1034,7 +1522,8 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
                           const int64_t *numels, int n_tensors, const tula_ags_hparams *hp,
                           void *stream) {
     Plan pl;
-    if (!hp || !g_small || !g_large || !valid_numels(numels, n_tensors, &pl)) return TULA_ERR_ARG;
+    if (!hp || !g_small || !g_large || !valid_numels(numels, n_tensors, 1, &pl))
+        return TULA_ERR_ARG;
     const int n = n_tensors;
     const bool per_elem = hp->granularity == TULA_SCALE_PER_ELEMENT;
     if (!per_elem && hp->granularity != TULA_SCALE_PER_TENSOR) return TULA_ERR_ARG;
@@ -1056,7 +1545,8 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
             dst[1] = g_large[p];
             dst[2] = hp->scale_elem[p];
         };
-        return launch_groups<kNP3>(k_scale_elem, n, numels, sc, hp->grid_ctas, s, fill);
+        return launch_streaming<kNP3>(k_scale_elem, n, numels, 4096, 0, sc, hp->grid_ctas, s,
+                                      fill);
     }
     int rc = check_ws(hp->workspace, hp->workspace_bytes, n, pl);
     if (rc) return rc;
@@ -1067,7 +1557,7 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
         dst[1] = nullptr;
         dst[2] = g_small[p];
     };
-    return run_reduce_k<1, false, false, true, true>(n, numels, sc, hp->grid_ctas, s, fill);
+    return run_reduce_k<1, false, false, true, true>(1, n, numels, sc, hp->grid_ctas, s, fill);
 }
 
 const char *tula_ags_error_string(int code) {
@@ -1139,15 +1629,15 @@ extern "C" int tula_ags_step_static_scratch(float *const *param_ptrs, float *con
                                             float weight_decay, const tula_ags_hparams *hp,
                                             void *stream) {
     Plan pl;
-    if (!hp || !valid_numels(numels, n_tensors, &pl)) return TULA_ERR_ARG;
+    if (!hp || !valid_numels(numels, n_tensors, hp->K, &pl)) return TULA_ERR_ARG;
     const WsLayout L = ws_layout(n_tensors, pl);
     if (L.total > kStaticScratchBytes) return TULA_ERR_SCRATCH_LIMIT;
     void *scratch = nullptr;
     int rc = static_scratch_address(&scratch);
     if (rc) return rc;
-    // The array keeps the last call's contents: zero the tickets, counters and
-    // branch flag (they precede the partial sums) before this call's kernels.
-    cudaError_t e = cudaMemsetAsync(scratch, 0, L.partials, static_cast<cudaStream_t>(stream));
+    // The array keeps the last call's contents: zero the counter, branch flag
+    // and error word (they precede the partial sums) before this call's kernels.
+    cudaError_t e = cudaMemsetAsync(scratch, 0, L.part1, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) {
         g_last_cuda = (int)e;
         return TULA_ERR_CUDA;

@@ -84,10 +84,14 @@ def lib() -> ctypes.CDLL:
     L.tula_ags_error_string.restype = ctypes.c_char_p
     L.tula_ags_last_cuda_error.restype = c_int
     L.tula_ags_launch_count.restype = ctypes.c_uint64
-    L.tula_ags_plan_chunks.argtypes = [i64p, c_int, i64p]
+    L.tula_ags_plan_chunks.argtypes = [i64p, c_int, c_int, i64p]
+    L.tula_ags_chunk_elems.argtypes = [c_int]
     L.tula_ags_chunk_elems.restype = c_int
+    L.tula_ags_workspace_error.argtypes = [c_void_p, c_size_t, i64p, c_int, c_int,
+                                           ctypes.POINTER(c_int)]
     for name in ("tula_ags_workspace_size", "tula_ags_step", "tula_layer_stats",
-                 "tula_ags_update_scale", "tula_ags_plan_chunks", "tula_ags_step_static_scratch"):
+                 "tula_ags_update_scale", "tula_ags_plan_chunks", "tula_ags_step_static_scratch",
+                 "tula_ags_workspace_error"):
         getattr(L, name).restype = c_int
     _lib = L
     return L
@@ -154,8 +158,19 @@ def tula_ags_launch_count() -> int:
     return lib().tula_ags_launch_count()
 
 
-def tula_ags_chunk_elems() -> int:
-    return lib().tula_ags_chunk_elems()
+def tula_ags_chunk_elems(streams: int) -> int:
+    return lib().tula_ags_chunk_elems(streams)
+
+
+def tula_ags_workspace_error(workspace: torch.Tensor, numels, K: int) -> int:
+    """Reads and clears the workspace's error word (synchronous): 0 = every wait completed."""
+    arr = (ctypes.c_int64 * max(1, len(numels)))(*[int(n) for n in numels])
+    out = c_int(0)
+    _check(lib().tula_ags_workspace_error(c_void_p(workspace.data_ptr()),
+                                          workspace.numel() * workspace.element_size(), arr,
+                                          len(numels), K, ctypes.byref(out)),
+           "tula_ags_workspace_error")
+    return out.value
 
 
 def tula_ags_default_hparams(K: int) -> tula_ags_hparams:
@@ -172,10 +187,10 @@ def tula_ags_workspace_size(numels, K: int = 1) -> int:
     return out.value
 
 
-def tula_ags_plan_chunks(numels) -> list[int]:
+def tula_ags_plan_chunks(numels, chunk_elems: int) -> list[int]:
     arr = (ctypes.c_int64 * max(1, len(numels)))(*[int(n) for n in numels])
     out = (ctypes.c_int64 * (len(numels) + 1))()
-    _check(lib().tula_ags_plan_chunks(arr, len(numels), out), "tula_ags_plan_chunks")
+    _check(lib().tula_ags_plan_chunks(arr, len(numels), chunk_elems, out), "tula_ags_plan_chunks")
     return list(out)
 
 
@@ -291,6 +306,10 @@ class AGSOptimizerStep:
         for i in range(3):
             ev = events[i] if events is not None else None
             self.hp.trace_events[i] = (ev.cuda_event if hasattr(ev, "cuda_event") else ev) or None
+
+    def error(self) -> int:
+        """Reads and clears the workspace error word (synchronous); 0 = all waits completed."""
+        return tula_ags_workspace_error(self.workspace, [t.numel() for t in self.params], self.K)
 
     def step(self, lr, momentum, weight_decay, refresh_scale=False, stream=None) -> None:
         self.hp.refresh_scale = 1 if refresh_scale else 0

@@ -39,25 +39,39 @@ def test_defaults_match_paper(lib):
         assert not hp.scale and not hp.state and not hp.workspace
 
 
-def test_plan_covers_every_element_once(lib):
-    C = T.tula_ags_chunk_elems()
+@pytest.mark.parametrize("streams", [1, 2, 3, 4, 9, 17, 18])
+def test_tile_fits_one_stage(lib, streams):
+    C = T.tula_ags_chunk_elems(streams)
+    assert C % 128 == 0 and 0 < C * 4 * streams <= 32 * 1024
+    assert C * 4 * streams > 32 * 1024 - 128 * 4 * streams  # the largest multiple of 128 that fits
+
+
+def test_tile_sizes_reject_bad_stream_counts(lib):
+    assert T.lib().tula_ags_chunk_elems(0) == T.TULA_ERR_ARG
+    assert T.lib().tula_ags_chunk_elems(19) == T.TULA_ERR_ARG
+
+
+@pytest.mark.parametrize("streams", [1, 9])
+def test_plan_covers_every_element_once(lib, streams):
+    C = T.tula_ags_chunk_elems(streams)
     numels = [0, 1, 3, C - 1, C, C + 1, 5 * C + 7, 64]
-    starts = T.tula_ags_plan_chunks(numels)
+    starts = T.tula_ags_plan_chunks(numels, C)
     assert starts[0] == 0
     for p, n in enumerate(numels):
         nch = starts[p + 1] - starts[p]
         assert nch == max(1, math.ceil(n / C))
         covered = sum(min(C, n - i * C) for i in range(nch)) if n else 0
         assert covered == n
-    assert starts == T.tula_ags_plan_chunks(numels)  # depends on the numels only
+    assert starts == T.tula_ags_plan_chunks(numels, C)  # depends on the numels only
 
 
-def test_workspace_size_grows_with_chunks(lib):
+def test_workspace_size_grows_with_tiles(lib):
     ps = W.param_set("resnet50")
     a = T.tula_ags_workspace_size(ps.numels, 8)
     b = T.tula_ags_workspace_size(ps.numels + [10 ** 8], 8)
     assert 0 < a < b and a % 256 == 0
-    assert T.tula_ags_workspace_size(ps.numels, 1) == a
+    # more replicas -> smaller reduction tiles -> more partial sums
+    assert T.tula_ags_workspace_size(ps.numels, 1) < a < T.tula_ags_workspace_size(ps.numels, 16)
 
 
 @pytest.mark.parametrize("numels,K", [([], 1), ([3, -1], 1), ([3], 0), ([3], 17)])
