@@ -48,7 +48,8 @@ extern "C" {
 
 #define TULA_OK 0
 #define TULA_ERR_ARG (-1)         /* NULL where a pointer is required, n_tensors < 1, K outside
-                                     [1, TULA_MAX_K], numel < 0, unaligned fp32 pointer, bad enum,
+                                     [1, TULA_MAX_K], numel < 0, a tensor above the size limit
+                                     (see tula_ags_step), unaligned fp32 pointer, bad enum,
                                      mom_ptrs NULL with momentum != 0, refresh with K == 1 */
 #define TULA_ERR_WORKSPACE (-2)   /* workspace NULL or smaller than tula_ags_workspace_size() */
 #define TULA_ERR_CUDA (-3)        /* a kernel launch failed; see tula_ags_last_cuda_error() */
@@ -135,7 +136,11 @@ int tula_ags_workspace_size(const int64_t *numels, int n_tensors, int K, size_t 
  *                          the other replicas are only read
  *   mom_ptrs[p]            momentum buffer m_p, device fp32, updated in place; mom_ptrs may be
  *                          NULL only when momentum == 0 (then w <- w - lr * d)
- *   numels[p] >= 0         element counts (0 = skipped)
+ *   numels[p] >= 0         element counts (0 = skipped); one tensor may span at most
+ *                          1,694,208 tiles of min(tula_ags_chunk_elems(K + 1),
+ *                          tula_ags_chunk_elems(4)) elements (K + 2 in place of K + 1 when
+ *                          K = 1): about 3.5e9 elements for K <= 2, 2.6e9 at K = 4, 1.5e9
+ *                          at K = 8, 6.5e8 at K = 16; a larger tensor gives TULA_ERR_ARG
  * Per element, with c the coefficient of the rule (Algorithm 1, Eq. 8):
  *   gbar = (((g_0 + g_1) + ...) + g_{K-1}) / K
  *   d    = c * gbar + weight_decay * w
@@ -182,8 +187,9 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
  * TULA_STATIC_SCRATCH_BYTES (16 MiB) inside this library.  Every GPU that loads the library holds
  * that array until the process exits.  hp->workspace and hp->workspace_bytes are ignored.
  *
- * Limit: the scratch a tensor list needs (tula_ags_workspace_size) is about 100 bytes per tensor
- * plus 6.1 bytes per 1000 parameters, e.g. 4096 tensors holding up to ~2.6e9 parameters.  A larger
+ * Limit: the scratch a tensor list needs (tula_ags_workspace_size) is about 110 bytes per tensor
+ * plus, per 1000 parameters, 13 bytes (K <= 2), 20 (K = 4), 31 (K = 8) or 67 (K = 16): e.g. 4096
+ * tensors holding up to ~1.3e9 parameters at K <= 2, ~5.4e8 at K = 8, ~2.5e8 at K = 16.  A larger
  * list is rejected with TULA_ERR_SCRATCH_LIMIT before anything is enqueued.
  *
  * Set-up: the first call on each device, with that device current, looks up the array's device

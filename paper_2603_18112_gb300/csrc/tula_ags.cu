@@ -1109,9 +1109,12 @@ bool valid_numels(const int64_t *numels, int n, int K, Plan *pl) {
     if (!numels || n < 1 || K < 1 || K > TULA_MAX_K) return false;
     const int t1 = chunk1_min(K), t2 = chunk2_min();
     Plan p;
+    // One tensor's tile partials must fit one combine table (see CombTable).
+    const long long max_tiles = (long long)CombTable::kMaxS * kSegTiles;
     for (int i = 0; i < n; ++i) {
         if (numels[i] < 0) return false;
         const long long a = tiles_of(numels[i], t1), b = tiles_of(numels[i], t2);
+        if (a > max_tiles || b > max_tiles) return false;
         p.c1 += a;
         p.c2 += b;
         p.s1 += segs_of(a);
@@ -1245,7 +1248,7 @@ int launch_combine(int n, const int64_t *numels, int chunk, const Scalars &sc, c
             ++cnt;
             ++p;
         }
-        if (cnt == 0) return TULA_ERR_UNSUPPORTED;  // one tensor with more segments than a table
+        if (cnt == 0) return TULA_ERR_ARG;  // excluded up front by valid_numels
         tab->n = cnt;
         tab->ns = ns;
         tab->sfirst[cnt] = ns;

@@ -81,6 +81,18 @@ def test_workspace_size_rejects(lib, numels, K):
     assert e.value.code == T.TULA_ERR_ARG
 
 
+@pytest.mark.parametrize("K", [1, 2, 4, 8, 16])
+def test_per_tensor_size_limit(lib, K):
+    """One tensor may span at most 6618 combine segments of 256 tiles (the
+    header's stated limit); the check happens before any launch."""
+    tile = min(T.tula_ags_chunk_elems(K + 2 if K == 1 else K + 1), T.tula_ags_chunk_elems(4))
+    limit = 1_694_208 * tile
+    assert T.tula_ags_workspace_size([limit], K) > 0
+    with pytest.raises(T.TulaError) as e:
+        T.tula_ags_workspace_size([limit + 1], K)
+    assert e.value.code == T.TULA_ERR_ARG
+
+
 def _call_step(lib, n=2, K=1, params=None, grads=None, moms=None, numels=None, hp=None,
                momentum=0.9):
     P = ctypes.c_void_p

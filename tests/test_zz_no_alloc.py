@@ -28,13 +28,13 @@ def test_rejects_tensor_lists_beyond_the_static_scratch():
     CUDA call (the pointers below are never dereferenced)."""
     B.build()
     lib = T.lib()
-    numels = [1 << 40]  # 2^40 elements = 2^26 chunks: far beyond 4 MiB of scratch
+    numels = [1 << 30] * 64  # 2^36 elements: ~0.9 GB of tile partials, far beyond 16 MiB
     assert T.tula_ags_workspace_size(numels, 1) > T.TULA_STATIC_SCRATCH_BYTES
     P = ctypes.c_void_p
-    ptrs = (P * 1)(0x100000)
+    ptrs = (P * 64)(*[0x100000 * (i + 1) for i in range(64)])
     hp = T.tula_ags_default_hparams(1)
     hp.scale, hp.state = 0x200000, 0x300000
-    rc = lib.tula_ags_step_static_scratch(ptrs, ptrs, ptrs, (ctypes.c_int64 * 1)(*numels), 1,
+    rc = lib.tula_ags_step_static_scratch(ptrs, ptrs, ptrs, (ctypes.c_int64 * 64)(*numels), 64,
                                           0.1, 0.9, 0.0, ctypes.byref(hp), None)
     assert rc == T.TULA_ERR_SCRATCH_LIMIT
     assert "static scratch" in T.tula_ags_error_string(rc)
