@@ -55,7 +55,9 @@ constexpr int kStageBytes = 32 * 1024;  // one tile of every stream
 constexpr int kStages = 6;              // ring depth (192 KB per CTA)
 constexpr int kConsumers = 3;           // consumer warps; consumer c owns stages c and c + 3
 constexpr int kThreads = 32 * (1 + kConsumers);
-constexpr int kSmemBytes = kStages * kStageBytes + 2 * kStages * 8;
+constexpr int kSmemBytes = kStages * kStageBytes + 2 * kStages * 8 + kStages * 4;
+constexpr int kDynTiles = 128;           // tiles per CTA from which a launch claims its tiles
+constexpr unsigned kClaim = 4;           // tiles per claim
 constexpr int kPend = 4;                // tiles whose warp reductions run together
 constexpr int kCombWarps = 4;           // k_combine: one warp per segment, 4 per CTA
 constexpr int kSegTiles = 256;          // tile partials per combine segment (8 per lane)
@@ -107,7 +109,7 @@ struct CombTable {
 
 struct Scalars {
     int K, rule, gran, force, refresh, mode, n_total, read_w;
-    int pow2K, pad0, pad1, pad2;
+    int pow2K, evict_first, pad1, pad2;  // evict_first: TMA loads ask L2 to drop their lines first
     float delta, eps, s_max, static_s, lars_trust, lr, mu, wd, invK, Kf;
     float *scale;
     double *state;
@@ -123,6 +125,7 @@ struct Scalars {
     double *spart2;  // [segment], pass 2
     double *tsum;    // [tensor][kTsum]: |gbar|^2, |g_0|^2, |w|^2
     float *cand;     // [tensor]: c_p of the scaled branch (AGS: the old gradscale)
+    unsigned *tiles; // [2 * pass]: next tile to claim, [2 * pass + 1]: CTAs finished
 };
 
 // ----------------------------------------------------------------------------
@@ -272,6 +275,21 @@ __device__ __forceinline__ void bulk_g2s(uint32_t dst, const void *src, uint32_t
         "l"(src), "r"(bytes), "r"(smem_addr(bar))
         : "memory");
 }
+// The same with an L2 cache policy for the source lines.
+__device__ __forceinline__ void bulk_g2s_hint(uint32_t dst, const void *src, uint32_t bytes,
+                                              uint64_t *bar, uint64_t policy) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1], %2, [%3], %4;" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(smem_addr(bar)), "l"(policy)
+        : "memory");
+}
+// L2 policy: these lines are the first to go.
+__device__ __forceinline__ uint64_t policy_evict_first() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
 
 __device__ __forceinline__ void report_timeout(const Scalars &sc) {
     atomicOr(sc.err, 1u);
@@ -365,41 +383,106 @@ struct TensorCache {
 // The producer: TMA bulk copies of each tile's streams into the stage ring
 // ----------------------------------------------------------------------------
 //
-// Tile j of this CTA (launch tile blockIdx.x + j * gridDim.x, or its mirror
-// image when `reverse`) goes to stage j % kStages and is consumed by consumer
-// warp j % kConsumers.  The whole producer warp works on a tile: lane i < ns
-// fetches stream i's pointer (role roles[i]) and issues that stream's copy, to
-// offset i * chunk floats of the stage, after lane 0 has posted the tile's
-// byte count on the stage's full barrier.
+// Two ways to deal a launch's tiles to its persistent CTAs:
+//  * round-robin (tile blockIdx.x + j * gridDim.x), for launches of fewer than
+//    kDynTiles tiles per CTA: nothing to claim, nothing to wait for;
+//  * claimed, for larger launches: the producer warp of each CTA takes kClaim
+//    consecutive tiles at a time from a global counter (ctr[0]), two claims
+//    ahead to hide the atomic's latency.  SMs do not stream at equal rates (on
+//    large launches the last CTA of a round-robin deal finished 15-30% after
+//    the median), so claiming lets the faster SMs take more tiles and the
+//    launch end with the memory system rather than with its slowest SM.  The
+//    last CTA to finish puts both counters (ctr[0], ctr[1]) back to zero.
+// Where a tile is processed never changes its result: each tile's partial sums
+// go to the tile's own slot and are combined in a fixed order later.  The j-th
+// tile of a CTA goes to stage j % kStages and is consumed by consumer warp
+// j % kConsumers; its launch tile index is left in stage_tile[stage] before the
+// stage's full barrier is armed (the barrier's release/acquire orders it), and
+// -1 there tells a consumer that no tile is left.  Lane i < ns of the producer
+// fetches stream i's pointer (role roles[i]) and issues that stream's copy to
+// offset i * chunk floats of the stage.  With `reverse` the order is mirrored
+// (pass 2 walks the tiles backwards, so it starts on what pass 1 left in L2).
+
+__device__ __forceinline__ unsigned claim_tiles(unsigned *ctr) { return atomicAdd(ctr, 1u); }
+
+// Round-robin tiles of this CTA (0 when the launch claims its tiles).
+__device__ __forceinline__ int static_tiles(int nc) {
+    const int g = (int)gridDim.x, b = (int)blockIdx.x;
+    if (nc >= kDynTiles * g) return 0;
+    return b < nc ? (nc - b + g - 1) / g : 0;
+}
+__device__ __forceinline__ bool claims_tiles(int nc) { return nc >= kDynTiles * (int)gridDim.x; }
+__device__ __forceinline__ int static_tile(int nc, int j, bool reverse) {
+    const int i = (int)blockIdx.x + j * (int)gridDim.x;
+    return reverse ? nc - 1 - i : i;
+}
 
 template <int NP, int NS>
 __device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
-                                        const int (&roles)[NS], int ns, int chunk, int ntiles,
-                                        bool reverse, uint32_t ring, uint64_t *full,
-                                        uint64_t *empty) {
+                                        const int (&roles)[NS], int ns, int chunk,
+                                        int js, unsigned *ctr, bool reverse, uint32_t ring,
+                                        uint64_t *full, uint64_t *empty, int *stage_tile) {
     const int lane = threadIdx.x & 31;
     const int role = lane < ns ? roles[lane] : 0;
+    const unsigned nc = (unsigned)tab.nc;
+    const bool claim = claims_tiles(tab.nc);
+    const bool hint = sc.evict_first != 0;
+    const uint64_t policy = policy_evict_first();
     TensorCache tc;
-    int issued = 0;
-    for (int j = 0; j < ntiles; ++j) {
+    unsigned next0 = 0u, next1 = 0u, used = 0u;  // claims in flight, tiles used of next0
+    if (claim && lane == 0) {
+        next0 = claim_tiles(ctr);
+        next1 = claim_tiles(ctr);
+    }
+    int issued = 0, ending = 0;
+    for (int j = 0; ending < kConsumers; ++j) {
         const int s = j % kStages;
+        unsigned i = nc;  // past the end: an end marker
+        if (j < js) {
+            i = blockIdx.x + (unsigned)j * gridDim.x;
+        } else if (claim) {
+            if (lane == 0) {
+                if (used == kClaim) {
+                    next0 = next1;
+                    used = 0u;
+                    // the counter only grows: no more claims once past the end
+                    if (next0 * kClaim < nc) next1 = claim_tiles(ctr);
+                }
+                i = next0 * kClaim + used;
+                ++used;
+            }
+            i = __shfl_sync(kFull, i, 0);
+        }
         if (j >= kStages) {
-            int ok = 1;
-            if (lane == 0) ok = mbar_wait(&empty[s], (uint32_t)((j / kStages - 1) & 1));
-            if (!__shfl_sync(kFull, ok, 0)) {
+            int w = 1;
+            if (lane == 0) w = mbar_wait(&empty[s], (uint32_t)((j / kStages - 1) & 1));
+            if (!__shfl_sync(kFull, w, 0)) {
                 if (lane == 0) report_timeout(sc);
                 break;
             }
         }
-        const int i = blockIdx.x + j * gridDim.x;
-        const int c = reverse ? tab.nc - 1 - i : i;
+        if (i >= nc) {  // one end marker per consumer warp
+            if (lane == 0) {
+                stage_tile[s] = -1;
+                mbar_arrive_tx(&full[s], 0u);
+            }
+            ++ending;
+            issued = j + 1;
+            continue;
+        }
+        const int c = reverse ? (int)(nc - 1u - i) : (int)i;
         const TilePos q = tc.at(tab, c, chunk, role, ns);
         const uint32_t bytes = 16u * (uint32_t)tc.nv;
-        if (lane == 0) mbar_arrive_tx(&full[s], bytes * (uint32_t)ns);
+        if (lane == 0) {
+            stage_tile[s] = c;
+            mbar_arrive_tx(&full[s], bytes * (uint32_t)ns);
+        }
         __syncwarp();
-        if (bytes && lane < ns)
-            bulk_g2s(ring + (uint32_t)s * kStageBytes + (uint32_t)(lane * chunk * 4),
-                     tc.mine + q.begin, bytes, &full[s]);
+        if (bytes && lane < ns) {
+            const uint32_t dst = ring + (uint32_t)s * kStageBytes + (uint32_t)(lane * chunk * 4);
+            if (hint) bulk_g2s_hint(dst, tc.mine + q.begin, bytes, &full[s], policy);
+            else bulk_g2s(dst, tc.mine + q.begin, bytes, &full[s]);
+        }
         issued = j + 1;
     }
     // Drain: never leave the CTA with a copy still writing into its shared memory.
@@ -408,14 +491,24 @@ __device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
             const int jl = s + ((issued - 1 - s) / kStages) * kStages;  // last tile on stage s
             if (!mbar_wait(&full[s], (uint32_t)((jl / kStages) & 1))) report_timeout(sc);
         }
+        // Every claim of this CTA is performed before it counts itself finished;
+        // the last CTA re-arms the counters for the next launch.
+        if (claim) {
+            __threadfence();
+            if (atomicAdd(ctr + 1, 1u) == gridDim.x - 1u) {
+                atomicExch(ctr, 0u);
+                atomicExch(ctr + 1, 0u);
+            }
+        }
     }
 }
 
-// Shared prologue of the streaming kernels: barrier init, tile count.
-__device__ __forceinline__ int ring_setup(unsigned char *smem, uint64_t *&full, uint64_t *&empty,
-                                          int nc) {
+// Shared prologue of the streaming kernels: barrier init.
+__device__ __forceinline__ void ring_setup(unsigned char *smem, uint64_t *&full, uint64_t *&empty,
+                                           int *&stage_tile) {
     full = reinterpret_cast<uint64_t *>(smem + kStages * kStageBytes);
     empty = full + kStages;
+    stage_tile = reinterpret_cast<int *>(empty + kStages);
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(&full[s], 1);
@@ -424,7 +517,18 @@ __device__ __forceinline__ int ring_setup(unsigned char *smem, uint64_t *&full, 
         mbar_fence_init();
     }
     __syncthreads();
-    return (int)blockIdx.x < nc ? (nc - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x : 0;
+}
+
+// A consumer's wait for its j-th tile: the launch tile index, -1 when no tile
+// is left, -2 when the wait ran out (reported).
+__device__ __forceinline__ int next_tile(const Scalars &sc, int j, uint64_t *full,
+                                         const int *stage_tile) {
+    const int s = j % kStages;
+    if (!mbar_wait(&full[s], (uint32_t)((j / kStages) & 1))) {
+        if ((threadIdx.x & 31) == 0) report_timeout(sc);
+        return -2;
+    }
+    return *reinterpret_cast<const volatile int *>(stage_tile + s);
 }
 
 // ----------------------------------------------------------------------------
@@ -586,7 +690,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     extern __shared__ __align__(128) unsigned char smem[];
     grid_dependency();
     uint64_t *full, *empty;
-    const int ntiles = ring_setup(smem, full, empty, tab.nc);
+    int *stage_tile;
+    ring_setup(smem, full, empty, stage_tile);
+    const int js = static_tiles(tab.nc);
     const uint32_t ring = smem_addr(smem);
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -598,18 +704,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (RW) roles[ns++] = KS;
     if (SS) roles[ns++] = KS + 1;
     if (warp == 0) {
-        produce<P1<KT>::NP, NSMAX>(tab, sc, roles, ns, chunk, ntiles, false, ring, full, empty);
+        produce<P1<KT>::NP, NSMAX>(tab, sc, roles, ns, chunk, js, sc.tiles, false, ring, full,
+                                   empty, stage_tile);
         return;
     }
     const int my_role = lane < ns ? roles[lane] : 0;
 
     const int cw = warp - 1;
     TensorCache tc;
-    for (int jb = cw; jb < ntiles; jb += kConsumers * kPend) {
+    bool stop = false;
+    for (int jb = cw; !stop; jb += kConsumers * kPend) {
         double pendd[PR ? kPend * kAcc : 1];
         float pendf[PR ? 1 : kPend * kAcc];
         int ptile[kPend];
-        bool stop = false;
 #pragma unroll
         for (int p = 0; p < kPend; ++p) {
             const int j = jb + p * kConsumers;
@@ -619,16 +726,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if constexpr (PR) pendd[p * kAcc + a] = 0.0;
                 else pendf[p * kAcc + a] = 0.f;
             }
-            if (stop || j >= ntiles) continue;
-            const int s = j % kStages;
-            const int c = blockIdx.x + j * gridDim.x;
-            const TilePos q = tc.at(tab, c, chunk, my_role, ns);
-            const float *const *ptr = tab.ptr[q.t];
-            if (!mbar_wait(&full[s], (uint32_t)((j / kStages) & 1))) {
-                if (lane == 0) report_timeout(sc);
+            if (stop) continue;
+            // A round-robin tile is located before its wait, a claimed one after.
+            int c = j < js ? static_tile(tab.nc, j, false) : -1;
+            TilePos q;
+            if (c >= 0) q = tc.at(tab, c, chunk, my_role, ns);
+            const int got = next_tile(sc, j, full, stage_tile);
+            if (got < 0) {
                 stop = true;
                 continue;
             }
+            if (c < 0) {
+                c = got;
+                q = tc.at(tab, c, chunk, my_role, ns);
+            }
+            const int s = j % kStages;
+            const float *const *ptr = tab.ptr[q.t];
             double accd[kAcc];
             float accf[kAcc];
             reduce_tile<KT, WM, RW, SS, PR>(ring + (uint32_t)s * kStageBytes, chunk, ptr, q,
@@ -898,7 +1011,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     extern __shared__ __align__(128) unsigned char smem[];
     grid_dependency();
     uint64_t *full, *empty;
-    const int ntiles = ring_setup(smem, full, empty, tab.nc);
+    int *stage_tile;
+    ring_setup(smem, full, empty, stage_tile);
+    const int js = static_tiles(tab.nc);
     const uint32_t ring = smem_addr(smem);
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -910,7 +1025,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     int roles[4] = {0, 1, 2, 3};
     if (!HM) roles[2] = 3;
     if (warp == 0) {
-        produce<kNP2, 4>(tab, sc, roles, ns, chunk, ntiles, true, ring, full, empty);
+        produce<kNP2, 4>(tab, sc, roles, ns, chunk, js, sc.tiles + 2, true, ring, full, empty,
+                         stage_tile);
         return;
     }
     const int my_role = lane < ns ? roles[lane] : 0;
@@ -922,31 +1038,41 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     TensorCache tc;
     const int cw = warp - 1;
-    for (int jb = cw; jb < ntiles; jb += kConsumers * kPend) {
+    int cand_t = -1;
+    float cand = 0.f;
+    bool stop = false;
+    for (int jb = cw; !stop; jb += kConsumers * kPend) {
         float pend[kPend];
         int ptile[kPend];
-        bool stop = false;
 #pragma unroll
         for (int p = 0; p < kPend; ++p) {
             const int j = jb + p * kConsumers;
             ptile[p] = -1;
             pend[p] = 0.f;
-            if (stop || j >= ntiles) continue;
+            if (stop) continue;
+            int c = j < js ? static_tile(tab.nc, j, true) : -1;
+            TilePos q;
+            if (c >= 0) q = tc.at(tab, c, chunk, my_role, ns);
+            const int got = next_tile(sc, j, full, stage_tile);
+            if (got < 0) {
+                stop = true;
+                continue;
+            }
+            if (c < 0) {
+                c = got;
+                q = tc.at(tab, c, chunk, my_role, ns);
+            }
             const int s = j % kStages;
-            const int c = tab.nc - 1 - ((int)blockIdx.x + j * (int)gridDim.x);
-            const TilePos q = tc.at(tab, c, chunk, my_role, ns);
             const float *const *ptr = tab.ptr[q.t];
             const int nv = tc.nv;
-            const float cand = sc.cand[q.tg];
+            if (q.tg != cand_t) {  // c_p changes only with the tensor
+                cand = sc.cand[q.tg];
+                cand_t = q.tg;
+            }
             const float ct = gated ? (scaled ? cand : 1.0f) : cand;
             if (sc.stats && q.c_in_t == 0 && lane == 0)
                 sc.stats[(size_t)q.tg * TULA_STATS_LEN + TULA_STAT_COEF] =
                     PE ? (scaled ? (double)NAN : 1.0) : (double)ct;
-            if (!mbar_wait(&full[s], (uint32_t)((j / kStages) & 1))) {
-                if (lane == 0) report_timeout(sc);
-                stop = true;
-                continue;
-            }
             const uint32_t stage = ring + (uint32_t)s * kStageBytes;
             float *wp = const_cast<float *>(ptr[1]) + q.begin;
             float *mp = HM ? const_cast<float *>(ptr[2]) + q.begin : nullptr;
@@ -1079,7 +1205,7 @@ struct Plan {
 // Workspace layout.  Every counter and flag precedes `part1`, so zeroing
 // [0, part1) clears all of them.
 struct WsLayout {
-    size_t done, flags, err, sctr1, sctr2, part1, part2, spart1, spart2, tsum, cand, total;
+    size_t done, flags, err, tiles, sctr1, sctr2, part1, part2, spart1, spart2, tsum, cand, total;
 };
 
 WsLayout ws_layout(int n_tensors, const Plan &pl) {
@@ -1093,6 +1219,7 @@ WsLayout ws_layout(int n_tensors, const Plan &pl) {
     L.done = take(sizeof(unsigned) * 4);
     L.flags = take(sizeof(int) * 4);
     L.err = take(sizeof(unsigned) * 4);
+    L.tiles = take(sizeof(unsigned) * 4);
     L.sctr1 = take(sizeof(unsigned) * (size_t)n_tensors);
     L.sctr2 = take(sizeof(unsigned) * (size_t)n_tensors);
     L.part1 = take(sizeof(double) * kAcc * (size_t)pl.c1);
@@ -1149,6 +1276,21 @@ int resident_ctas(const void *kernel, int threads, int smem) {
     const int ctas = std::max(1, sms * std::max(per, 1));
     cache.push_back({kernel, dev, ctas});
     return ctas;
+}
+
+// L2 capacity of the current device in bytes (cached; 0 if unknown).
+long long l2_bytes() {
+    static std::mutex mu;
+    static std::vector<std::pair<int, long long>> cache;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    std::lock_guard<std::mutex> lock(mu);
+    for (const auto &e : cache)
+        if (e.first == dev) return e.second;
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrL2CacheSize, dev) != cudaSuccess) v = 0;
+    cache.emplace_back(dev, (long long)v);
+    return v;
 }
 
 // Launch with programmatic stream serialization: the kernel may begin while
@@ -1288,6 +1430,7 @@ Scalars make_scalars(const tula_ags_hparams *hp, int K, int n, void *ws, const W
     sc.done = reinterpret_cast<unsigned *>(b + L.done);
     sc.flags = reinterpret_cast<int *>(b + L.flags);
     sc.err = reinterpret_cast<unsigned *>(b + L.err);
+    sc.tiles = reinterpret_cast<unsigned *>(b + L.tiles);
     sc.sctr1 = reinterpret_cast<unsigned *>(b + L.sctr1);
     sc.sctr2 = reinterpret_cast<unsigned *>(b + L.sctr2);
     sc.part1 = reinterpret_cast<double *>(b + L.part1);
@@ -1441,6 +1584,12 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
     Scalars sc = make_scalars(hp, K, n, hp->workspace, L, kModeStep);
     const bool lars = hp->rule == TULA_RULE_LARS;
     sc.read_w = lars ? 1 : 0;
+    // When the mean fits in L2, the replica loads of pass 1 are marked to leave
+    // L2 first, so that pass 2 (which walks the tiles backwards) finds much of
+    // the mean still there.  For larger models the mark only costs bandwidth.
+    long long n_total = 0;
+    for (int p = 0; p < n; ++p) n_total += numels[p];
+    sc.evict_first = (K > 1 && 4 * n_total <= l2_bytes()) ? 1 : 0;
     sc.lr = lr;
     sc.mu = momentum;
     sc.wd = weight_decay;
