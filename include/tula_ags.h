@@ -116,8 +116,13 @@ typedef struct tula_ags_hparams {
     size_t workspace_bytes;
     int grid_ctas;                /* CTAs per launch; 0 = one wave of resident CTAs (results do
                                      not depend on it) */
-    void *trace_events[3];        /* optional cudaEvent_t, recorded on `stream` before the
-                                     reduction pass, between the passes, after the update pass */
+    void *trace_events[5];        /* optional cudaEvent_t (NULL = none), recorded on `stream`:
+                                     [0] before the reduction kernel(s), [1] after them,
+                                     [2] after the pass-1 combine (before the update kernel),
+                                     [3] after the update kernel(s), [4] after the pass-2
+                                     combine (the end of the step).  A recorded event keeps the
+                                     next kernel from starting early, so steps that record
+                                     events run slightly slower. */
 } tula_ags_hparams;
 
 /* Fills *hp with the paper's defaults for K replicas: AGS, per tensor, automatic branch,
@@ -137,10 +142,10 @@ int tula_ags_workspace_size(const int64_t *numels, int n_tensors, int K, size_t 
  *   mom_ptrs[p]            momentum buffer m_p, device fp32, updated in place; mom_ptrs may be
  *                          NULL only when momentum == 0 (then w <- w - lr * d)
  *   numels[p] >= 0         element counts (0 = skipped); one tensor may span at most
- *                          1,694,208 tiles of min(tula_ags_chunk_elems(K + 1),
- *                          tula_ags_chunk_elems(4)) elements (K + 2 in place of K + 1 when
- *                          K = 1): about 3.5e9 elements for K <= 2, 2.6e9 at K = 4, 1.5e9
- *                          at K = 8, 6.5e8 at K = 16; a larger tensor gives TULA_ERR_ARG
+ *                          1,694,208 tiles of min(tula_ags_chunk_elems(1, K + 1),
+ *                          tula_ags_chunk_elems(2, 4)) elements (K + 2 in place of K + 1
+ *                          when K = 1): about 2.6e9 elements for K <= 4, 1.5e9 at K = 8,
+ *                          6.5e8 at K = 16; a larger tensor gives TULA_ERR_ARG
  * Per element, with c the coefficient of the rule (Algorithm 1, Eq. 8):
  *   gbar = (((g_0 + g_1) + ...) + g_{K-1}) / K
  *   d    = c * gbar + weight_decay * w
@@ -216,12 +221,13 @@ int tula_ags_last_cuda_error(void);
 uint64_t tula_ags_launch_count(void);
 
 /*
- * Elements per tile (work item) of a pass that streams `streams` tensors through shared memory
- * (the reduction pass: K replicas [+ w] [+ g_small]; the update pass: gbar, w [+ m] [+ per-element
- * scale]): one tile of every stream fills one 32 KB stage.  A multiple of 128; TULA_ERR_ARG when
- * streams is outside [1, TULA_MAX_K + 2].
+ * Elements per tile (work item) of a pass that streams `streams` tensors through shared memory:
+ * pass 1, the reduction (K replicas [+ w] [+ g_small]; one tile of every stream fills a 32 KB
+ * stage), or pass 2, the update (gbar, w [+ m] [+ per-element scale]; a 24 KB stage).  A multiple
+ * of 128; TULA_ERR_ARG for another pass or when streams is outside [1, TULA_MAX_K + 2] (pass 1)
+ * or [1, 4] (pass 2).
  */
-int tula_ags_chunk_elems(int streams);
+int tula_ags_chunk_elems(int pass, int streams);
 
 /*
  * Host-only view of the work decomposition: tensor p is split into

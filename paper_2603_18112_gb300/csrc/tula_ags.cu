@@ -51,11 +51,30 @@
 
 namespace {
 
-constexpr int kStageBytes = 32 * 1024;  // one tile of every stream
-constexpr int kStages = 6;              // ring depth (192 KB per CTA)
-constexpr int kConsumers = 3;           // consumer warps; consumer c owns stages c and c + 3
-constexpr int kThreads = 32 * (1 + kConsumers);
-constexpr int kSmemBytes = kStages * kStageBytes + 2 * kStages * 8 + kStages * 4;
+// A stage ring: kStages shared-memory stages of kStageBytes each (one tile of
+// every stream), one producer warp and kConsumers consumer warps.  A consumer
+// must own whole stages: the tile it waits for on a stage is then always the
+// one after its own previous tile there, so a parity wait never sees a phase
+// two ahead.
+template <int StageKB, int Stages, int Consumers>
+struct Ring {
+    static constexpr int kStageBytes = StageKB * 1024;
+    static constexpr int kStages = Stages;
+    static constexpr int kConsumers = Consumers;
+    static constexpr int kThreads = 32 * (1 + Consumers);
+    static constexpr int kSmemBytes = Stages * kStageBytes + 2 * Stages * 8 + Stages * 4;
+    static_assert(Stages % Consumers == 0, "consumers own whole stages");
+    static_assert(kSmemBytes <= 227 * 1024, "one CTA per SM");
+    // Elements per tile when `streams` tensors share one stage (multiple of 128).
+    __host__ __device__ static constexpr int tile_elems(int streams) {
+        return (kStageBytes / (4 * streams)) / 128 * 128;
+    }
+};
+// Pass 1 streams K (+1, +2) tensors and little arithmetic: large copies, few
+// consumers.  Pass 2 does ~11 flops per element over 3-4 streams: its
+// consumers, not HBM, set the pace with three warps, so it runs four.
+using Ring1 = Ring<32, 6, 3>;
+using Ring2 = Ring<24, 8, 4>;
 constexpr int kDynTiles = 128;           // tiles per CTA from which a launch claims its tiles
 constexpr unsigned kClaim = 4;           // tiles per claim
 constexpr int kPend = 4;                // tiles whose warp reductions run together
@@ -69,10 +88,6 @@ constexpr uint32_t kSpinLimit = 1u << 22;  // bound on every mbarrier wait (>= 1
 
 enum Mode { kModeStep = 0, kModeStats = 1, kModeScale = 2, kModeUpdate = 3 };
 
-// Elements per tile when `streams` tensors share one 32 KB stage (multiple of 128).
-__host__ __device__ constexpr int tile_elems(int streams) {
-    return (kStageBytes / (4 * streams)) / 128 * 128;
-}
 
 // ----------------------------------------------------------------------------
 // Launch tables (kernel parameters)
@@ -86,7 +101,8 @@ struct Table {
     int c0;     // global index of its first tile
     int nc;     // tiles in this launch
     int chunk;  // elements per tile
-    int pad[3];
+    int first;  // 1 for the first launch of the pass (in issue order)
+    int pad[2];
     long long numel[kMaxT];
     int cstart[kMaxT + 1];  // first tile of each tensor, relative to c0; cstart[n] = nc
     const float *ptr[kMaxT][NP];
@@ -220,9 +236,13 @@ __device__ __forceinline__ void warp_sums(float (&v)[R]) {
 
 // Wait for the grids this one depends on to complete and their memory to be
 // visible, then let the next grid in the stream begin launching.
-__device__ __forceinline__ void grid_dependency() {
-    asm volatile("griddepcontrol.wait;" ::: "memory");
+__device__ __forceinline__ void grid_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_launch_dependents() {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void grid_dependency() {
+    grid_wait();
+    grid_launch_dependents();
 }
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p) {
@@ -417,7 +437,7 @@ __device__ __forceinline__ int static_tile(int nc, int j, bool reverse) {
     return reverse ? nc - 1 - i : i;
 }
 
-template <int NP, int NS>
+template <typename R, int NP, int NS>
 __device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
                                         const int (&roles)[NS], int ns, int chunk,
                                         int js, unsigned *ctr, bool reverse, uint32_t ring,
@@ -435,8 +455,8 @@ __device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
         next1 = claim_tiles(ctr);
     }
     int issued = 0, ending = 0;
-    for (int j = 0; ending < kConsumers; ++j) {
-        const int s = j % kStages;
+    for (int j = 0; ending < R::kConsumers; ++j) {
+        const int s = j % R::kStages;
         unsigned i = nc;  // past the end: an end marker
         if (j < js) {
             i = blockIdx.x + (unsigned)j * gridDim.x;
@@ -453,9 +473,9 @@ __device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
             }
             i = __shfl_sync(kFull, i, 0);
         }
-        if (j >= kStages) {
+        if (j >= R::kStages) {
             int w = 1;
-            if (lane == 0) w = mbar_wait(&empty[s], (uint32_t)((j / kStages - 1) & 1));
+            if (lane == 0) w = mbar_wait(&empty[s], (uint32_t)((j / R::kStages - 1) & 1));
             if (!__shfl_sync(kFull, w, 0)) {
                 if (lane == 0) report_timeout(sc);
                 break;
@@ -479,7 +499,7 @@ __device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
         }
         __syncwarp();
         if (bytes && lane < ns) {
-            const uint32_t dst = ring + (uint32_t)s * kStageBytes + (uint32_t)(lane * chunk * 4);
+            const uint32_t dst = ring + (uint32_t)s * R::kStageBytes + (uint32_t)(lane * chunk * 4);
             if (hint) bulk_g2s_hint(dst, tc.mine + q.begin, bytes, &full[s], policy);
             else bulk_g2s(dst, tc.mine + q.begin, bytes, &full[s]);
         }
@@ -487,9 +507,9 @@ __device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
     }
     // Drain: never leave the CTA with a copy still writing into its shared memory.
     if (lane == 0) {
-        for (int s = 0; s < kStages && s < issued; ++s) {
-            const int jl = s + ((issued - 1 - s) / kStages) * kStages;  // last tile on stage s
-            if (!mbar_wait(&full[s], (uint32_t)((jl / kStages) & 1))) report_timeout(sc);
+        for (int s = 0; s < R::kStages && s < issued; ++s) {
+            const int jl = s + ((issued - 1 - s) / R::kStages) * R::kStages;  // last tile on stage s
+            if (!mbar_wait(&full[s], (uint32_t)((jl / R::kStages) & 1))) report_timeout(sc);
         }
         // Every claim of this CTA is performed before it counts itself finished;
         // the last CTA re-arms the counters for the next launch.
@@ -504,13 +524,14 @@ __device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
 }
 
 // Shared prologue of the streaming kernels: barrier init.
+template <typename R>
 __device__ __forceinline__ void ring_setup(unsigned char *smem, uint64_t *&full, uint64_t *&empty,
                                            int *&stage_tile) {
-    full = reinterpret_cast<uint64_t *>(smem + kStages * kStageBytes);
-    empty = full + kStages;
-    stage_tile = reinterpret_cast<int *>(empty + kStages);
+    full = reinterpret_cast<uint64_t *>(smem + R::kStages * R::kStageBytes);
+    empty = full + R::kStages;
+    stage_tile = reinterpret_cast<int *>(empty + R::kStages);
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) {
+        for (int s = 0; s < R::kStages; ++s) {
             mbar_init(&full[s], 1);
             mbar_init(&empty[s], 1);
         }
@@ -521,10 +542,11 @@ __device__ __forceinline__ void ring_setup(unsigned char *smem, uint64_t *&full,
 
 // A consumer's wait for its j-th tile: the launch tile index, -1 when no tile
 // is left, -2 when the wait ran out (reported).
+template <typename R>
 __device__ __forceinline__ int next_tile(const Scalars &sc, int j, uint64_t *full,
                                          const int *stage_tile) {
-    const int s = j % kStages;
-    if (!mbar_wait(&full[s], (uint32_t)((j / kStages) & 1))) {
+    const int s = j % R::kStages;
+    if (!mbar_wait(&full[s], (uint32_t)((j / R::kStages) & 1))) {
         if ((threadIdx.x & 31) == 0) report_timeout(sc);
         return -2;
     }
@@ -592,7 +614,7 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
     float fg = 0.f, fs = 0.f, fw = 0.f;   // fp32 sums (not PR)
 
     if constexpr (KT > 0) {
-        constexpr int CH = tile_elems(KT + (RW ? 1 : 0) + (SS ? 1 : 0));
+        constexpr int CH = Ring1::tile_elems(KT + (RW ? 1 : 0) + (SS ? 1 : 0));
         constexpr int COLS = CH / 128;  // float4 columns per lane of a full tile
         if (nv == CH / 4) {
             // Full tile: every lane has COLS columns; all loads of a column issue together.
@@ -683,7 +705,7 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
 }
 
 template <int KT, bool WM, bool RW, bool SS, bool PR>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(Ring1::kThreads, 1)
     k_reduce(const __grid_constant__ Table<P1<KT>::NP> tab, const __grid_constant__ Scalars sc) {
     constexpr int KS = P1<KT>::KS;
     constexpr int NSMAX = KS + 2;
@@ -691,7 +713,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     grid_dependency();
     uint64_t *full, *empty;
     int *stage_tile;
-    ring_setup(smem, full, empty, stage_tile);
+    ring_setup<Ring1>(smem, full, empty, stage_tile);
     const int js = static_tiles(tab.nc);
     const uint32_t ring = smem_addr(smem);
     const int warp = threadIdx.x >> 5;
@@ -704,7 +726,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (RW) roles[ns++] = KS;
     if (SS) roles[ns++] = KS + 1;
     if (warp == 0) {
-        produce<P1<KT>::NP, NSMAX>(tab, sc, roles, ns, chunk, js, sc.tiles, false, ring, full,
+        produce<Ring1, P1<KT>::NP, NSMAX>(tab, sc, roles, ns, chunk, js, sc.tiles, false, ring, full,
                                    empty, stage_tile);
         return;
     }
@@ -713,13 +735,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int cw = warp - 1;
     TensorCache tc;
     bool stop = false;
-    for (int jb = cw; !stop; jb += kConsumers * kPend) {
+    for (int jb = cw; !stop; jb += Ring1::kConsumers * kPend) {
         double pendd[PR ? kPend * kAcc : 1];
         float pendf[PR ? 1 : kPend * kAcc];
         int ptile[kPend];
 #pragma unroll
         for (int p = 0; p < kPend; ++p) {
-            const int j = jb + p * kConsumers;
+            const int j = jb + p * Ring1::kConsumers;
             ptile[p] = -1;
 #pragma unroll
             for (int a = 0; a < kAcc; ++a) {
@@ -731,7 +753,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             int c = j < js ? static_tile(tab.nc, j, false) : -1;
             TilePos q;
             if (c >= 0) q = tc.at(tab, c, chunk, my_role, ns);
-            const int got = next_tile(sc, j, full, stage_tile);
+            const int got = next_tile<Ring1>(sc, j, full, stage_tile);
             if (got < 0) {
                 stop = true;
                 continue;
@@ -740,11 +762,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 c = got;
                 q = tc.at(tab, c, chunk, my_role, ns);
             }
-            const int s = j % kStages;
+            const int s = j % Ring1::kStages;
             const float *const *ptr = tab.ptr[q.t];
             double accd[kAcc];
             float accf[kAcc];
-            reduce_tile<KT, WM, RW, SS, PR>(ring + (uint32_t)s * kStageBytes, chunk, ptr, q,
+            reduce_tile<KT, WM, RW, SS, PR>(ring + (uint32_t)s * Ring1::kStageBytes, chunk, ptr, q,
                                             tc.nv, sc, accd, accf);
             __syncwarp();
             if (lane == 0) mbar_arrive(&empty[s]);
@@ -1006,31 +1028,43 @@ __device__ __forceinline__ float update4(float4 g4, float4 w4, float4 m4, float4
 }
 
 template <bool HM, bool PE, bool SW>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(Ring2::kThreads, 1)
     k_update(const __grid_constant__ Table<kNP2> tab, const __grid_constant__ Scalars sc) {
     extern __shared__ __align__(128) unsigned char smem[];
-    grid_dependency();
+    // The first launch of the pass follows the pass-1 combine, which starts it
+    // once the reduction kernel has completed (the combine's own wait).  gbar, w
+    // and m are then final, so the producer streams tiles in while the combine
+    // still runs; the branch and the coefficients the consumers apply are the
+    // combine's output, so every consumer waits for its completion first.  The
+    // whole CTA waits per element (the producer's stream count depends on the
+    // branch) and in later launches of the pass (which share the tile counter
+    // with the launch before).
+    grid_launch_dependents();
+    const bool early = !PE && tab.first;
+    if (!early) grid_wait();
     uint64_t *full, *empty;
     int *stage_tile;
-    ring_setup(smem, full, empty, stage_tile);
+    ring_setup<Ring2>(smem, full, empty, stage_tile);
     const int js = static_tiles(tab.nc);
     const uint32_t ring = smem_addr(smem);
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int chunk = tab.chunk;
+    int roles[4] = {0, 1, 2, 3};
+    if (!HM) roles[2] = 3;
+    if (warp == 0) {
+        const bool se = PE && sc.flags[0];
+        produce<Ring2, kNP2, 4>(tab, sc, roles, 2 + (HM ? 1 : 0) + (se ? 1 : 0), chunk, js, sc.tiles + 2,
+                         true, ring, full, empty, stage_tile);
+        return;
+    }
+    if (early) grid_wait();
     const int scaled = sc.flags[0];
     const bool gated = sc.rule == TULA_RULE_AGS || sc.rule == TULA_RULE_STATIC;
     const bool use_se = PE && scaled;
     const int ns = 2 + (HM ? 1 : 0) + (use_se ? 1 : 0);
-    int roles[4] = {0, 1, 2, 3};
-    if (!HM) roles[2] = 3;
-    if (warp == 0) {
-        produce<kNP2, 4>(tab, sc, roles, ns, chunk, js, sc.tiles + 2, true, ring, full, empty,
-                         stage_tile);
-        return;
-    }
     const int my_role = lane < ns ? roles[lane] : 0;
-    constexpr int CH = tile_elems(2 + (HM ? 1 : 0) + (PE ? 1 : 0));
+    constexpr int CH = Ring2::tile_elems(2 + (HM ? 1 : 0) + (PE ? 1 : 0));
     constexpr int COLS = CH / 128;
     const uint32_t w_off = (uint32_t)(CH * 4);
     const uint32_t m_off = (uint32_t)(2 * CH * 4);
@@ -1041,19 +1075,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     int cand_t = -1;
     float cand = 0.f;
     bool stop = false;
-    for (int jb = cw; !stop; jb += kConsumers * kPend) {
+    for (int jb = cw; !stop; jb += Ring2::kConsumers * kPend) {
         float pend[kPend];
         int ptile[kPend];
 #pragma unroll
         for (int p = 0; p < kPend; ++p) {
-            const int j = jb + p * kConsumers;
+            const int j = jb + p * Ring2::kConsumers;
             ptile[p] = -1;
             pend[p] = 0.f;
             if (stop) continue;
             int c = j < js ? static_tile(tab.nc, j, true) : -1;
             TilePos q;
             if (c >= 0) q = tc.at(tab, c, chunk, my_role, ns);
-            const int got = next_tile(sc, j, full, stage_tile);
+            const int got = next_tile<Ring2>(sc, j, full, stage_tile);
             if (got < 0) {
                 stop = true;
                 continue;
@@ -1062,7 +1096,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 c = got;
                 q = tc.at(tab, c, chunk, my_role, ns);
             }
-            const int s = j % kStages;
+            const int s = j % Ring2::kStages;
             const float *const *ptr = tab.ptr[q.t];
             const int nv = tc.nv;
             if (q.tg != cand_t) {  // c_p changes only with the tensor
@@ -1073,7 +1107,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (sc.stats && q.c_in_t == 0 && lane == 0)
                 sc.stats[(size_t)q.tg * TULA_STATS_LEN + TULA_STAT_COEF] =
                     PE ? (scaled ? (double)NAN : 1.0) : (double)ct;
-            const uint32_t stage = ring + (uint32_t)s * kStageBytes;
+            const uint32_t stage = ring + (uint32_t)s * Ring2::kStageBytes;
             float *wp = const_cast<float *>(ptr[1]) + q.begin;
             float *mp = HM ? const_cast<float *>(ptr[2]) + q.begin : nullptr;
             const float4 cdef = PE ? make_float4(1.f, 1.f, 1.f, 1.f) : make_float4(ct, ct, ct, ct);
@@ -1151,12 +1185,14 @@ __device__ __forceinline__ float scale1(float gs, float gl, const Scalars &sc) {
     return fminf(fabsf(__fdiv_rn(gs, __fadd_rn(gl, sc.eps))), sc.s_max);
 }
 
-__global__ void __launch_bounds__(kThreads)
+constexpr int kScaleThreads = 128;
+
+__global__ void __launch_bounds__(kScaleThreads)
     k_scale_elem(const __grid_constant__ Table<kNP3> tab, const __grid_constant__ Scalars sc) {
     grid_dependency();
     const int lane = threadIdx.x & 31;
-    const int warp = (int)((blockIdx.x * (unsigned)kThreads + threadIdx.x) >> 5);
-    const int nwarps = (int)((gridDim.x * (unsigned)kThreads) >> 5);
+    const int warp = (int)((blockIdx.x * (unsigned)kScaleThreads + threadIdx.x) >> 5);
+    const int nwarps = (int)((gridDim.x * (unsigned)kScaleThreads) >> 5);
     Walker walk;
     for (int c = warp; c < tab.nc; c += nwarps) {
         const TilePos q = locate(tab, c, walk.to(tab, c), tab.chunk);
@@ -1191,8 +1227,10 @@ inline int replica_slot(int K) {
 }
 
 // Tile sizes: the smallest a pass can use for K replicas sizes the workspace.
-inline int chunk1(int K, bool rw, bool ss) { return tile_elems(K + (rw ? 1 : 0) + (ss ? 1 : 0)); }
-inline int chunk2(bool hm, bool pe) { return tile_elems(2 + (hm ? 1 : 0) + (pe ? 1 : 0)); }
+inline int chunk1(int K, bool rw, bool ss) {
+    return Ring1::tile_elems(K + (rw ? 1 : 0) + (ss ? 1 : 0));
+}
+inline int chunk2(bool hm, bool pe) { return Ring2::tile_elems(2 + (hm ? 1 : 0) + (pe ? 1 : 0)); }
 inline int chunk1_min(int K) { return chunk1(K, true, K == 1); }
 inline int chunk2_min() { return chunk2(true, true); }
 
@@ -1323,11 +1361,11 @@ int launch_pdl(void (*kernel)(KArgs...), int grid, int threads, int smem, cudaSt
 // launches `kernel` once per block (in reverse block order when `reverse`).
 // fill(p, ptrs) writes tensor p's pointers.
 template <int NP, typename Kernel, typename Fill>
-int launch_streaming(Kernel kernel, int n, const int64_t *numels, int chunk, int smem,
-                     const Scalars &sc, int grid_override, cudaStream_t stream, Fill fill,
-                     bool reverse = false) {
+int launch_streaming(Kernel kernel, int n, const int64_t *numels, int chunk, int threads,
+                     int smem, const Scalars &sc, int grid_override, cudaStream_t stream,
+                     Fill fill, bool reverse = false) {
     using T = Table<NP>;
-    const int grid_cap = resident_ctas((const void *)kernel, kThreads, smem);
+    const int grid_cap = resident_ctas((const void *)kernel, threads, smem);
     if (grid_cap <= 0) {
         g_last_cuda = (int)cudaGetLastError();
         return TULA_ERR_CUDA;
@@ -1357,10 +1395,11 @@ int launch_streaming(Kernel kernel, int n, const int64_t *numels, int chunk, int
         tabs.push_back(std::move(tab));
     }
     if (reverse) std::reverse(tabs.begin(), tabs.end());
+    tabs.front()->first = 1;
     for (const auto &tab : tabs) {
         int grid = grid_override > 0 ? grid_override : grid_cap;
         grid = std::max(1, std::min(grid, tab->nc));
-        const int rc = launch_pdl(kernel, grid, kThreads, smem, stream, *tab, sc);
+        const int rc = launch_pdl(kernel, grid, threads, smem, stream, *tab, sc);
         if (rc) return rc;
     }
     return TULA_OK;
@@ -1442,27 +1481,33 @@ Scalars make_scalars(const tula_ags_hparams *hp, int K, int n, void *ws, const W
     return sc;
 }
 
+void record(void *ev, cudaStream_t s) {
+    if (ev) cudaEventRecord(static_cast<cudaEvent_t>(ev), s);
+}
+
 // Pass 1 (+ its combine) dispatched over the compile-time replica count.
 template <int KT, bool WM, bool RW, bool SS, bool PR, typename Fill>
 int run_reduce_k(int K, int n, const int64_t *numels, const Scalars &sc, int grid, cudaStream_t s,
-                 Fill fill) {
+                 Fill fill, void *mid_event) {
     const int chunk = chunk1(K, RW, SS);
     int rc = launch_streaming<P1<KT>::NP>(k_reduce<KT, WM, RW, SS, PR>, n, numels, chunk,
-                                          kSmemBytes, sc, grid, s, fill);
+                                          Ring1::kThreads, Ring1::kSmemBytes, sc, grid, s,
+                                          fill);
     if (rc) return rc;
+    record(mid_event, s);
     return launch_combine<kAcc>(n, numels, chunk, sc, s);
 }
 
 template <bool WM, bool RW, bool SS, bool PR, typename Fill>
 int run_reduce(int K, int n, const int64_t *numels, const Scalars &sc, int grid, cudaStream_t s,
-               Fill fill) {
+               Fill fill, void *mid_event = nullptr) {
     switch (K) {
-    case 1: return run_reduce_k<1, false, RW, SS, PR>(K, n, numels, sc, grid, s, fill);
-    case 2: return run_reduce_k<2, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill);
-    case 4: return run_reduce_k<4, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill);
-    case 8: return run_reduce_k<8, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill);
-    case 16: return run_reduce_k<16, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill);
-    default: return run_reduce_k<0, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill);
+    case 1: return run_reduce_k<1, false, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event);
+    case 2: return run_reduce_k<2, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event);
+    case 4: return run_reduce_k<4, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event);
+    case 8: return run_reduce_k<8, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event);
+    case 16: return run_reduce_k<16, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event);
+    default: return run_reduce_k<0, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event);
     }
 }
 
@@ -1473,9 +1518,6 @@ int check_ws(void *ws, size_t bytes, int n, const Plan &pl) {
     return TULA_OK;
 }
 
-void record(void *ev, cudaStream_t s) {
-    if (ev) cudaEventRecord(static_cast<cudaEvent_t>(ev), s);
-}
 
 }  // namespace
 
@@ -1507,9 +1549,11 @@ int tula_ags_workspace_size(const int64_t *numels, int n_tensors, int K, size_t 
     return TULA_OK;
 }
 
-int tula_ags_chunk_elems(int streams) {
+int tula_ags_chunk_elems(int pass, int streams) {
     if (streams < 1 || streams > TULA_MAX_K + 2) return TULA_ERR_ARG;
-    return tile_elems(streams);
+    if (pass == 1) return Ring1::tile_elems(streams);
+    if (pass == 2 && streams <= 4) return Ring2::tile_elems(streams);
+    return TULA_ERR_ARG;
 }
 
 int tula_ags_plan_chunks(const int64_t *numels, int n_tensors, int chunk_elems,
@@ -1603,13 +1647,16 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
     record(hp->trace_events[0], s);
     // Norms feeding a coefficient (LARS, UpdateGradScale) are taken precisely.
     if (lars)
-        rc = run_reduce<true, true, false, true>(K, n, numels, sc, hp->grid_ctas, s, fill1);
+        rc = run_reduce<true, true, false, true>(K, n, numels, sc, hp->grid_ctas, s, fill1,
+                                                 hp->trace_events[1]);
     else if (hp->refresh_scale)
-        rc = run_reduce<true, false, false, true>(K, n, numels, sc, hp->grid_ctas, s, fill1);
+        rc = run_reduce<true, false, false, true>(K, n, numels, sc, hp->grid_ctas, s, fill1,
+                                                  hp->trace_events[1]);
     else
-        rc = run_reduce<true, false, false, false>(K, n, numels, sc, hp->grid_ctas, s, fill1);
+        rc = run_reduce<true, false, false, false>(K, n, numels, sc, hp->grid_ctas, s, fill1,
+                                                   hp->trace_events[1]);
     if (rc) return rc;
-    record(hp->trace_events[1], s);
+    record(hp->trace_events[2], s);
 
     auto fill2 = [&](int p, const float **dst) {
         dst[0] = grad_ptrs[p];
@@ -1621,9 +1668,9 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
     const bool sw = hp->layer_stats != nullptr && !lars;
     const int c2 = chunk2(hm, per_elem);
     sc.mode = kModeUpdate;
-#define TULA_UPD(HM, PE, SW)                                                                       \
-    launch_streaming<kNP2>(k_update<HM, PE, SW>, n, numels, c2, kSmemBytes, sc, hp->grid_ctas, s, \
-                           fill2, true)
+#define TULA_UPD(HM, PE, SW)                                                                \
+    launch_streaming<kNP2>(k_update<HM, PE, SW>, n, numels, c2, Ring2::kThreads,             \
+                           Ring2::kSmemBytes, sc, hp->grid_ctas, s, fill2, true)
     if (hm) {
         if (per_elem) rc = sw ? TULA_UPD(true, true, true) : TULA_UPD(true, true, false);
         else rc = sw ? TULA_UPD(true, false, true) : TULA_UPD(true, false, false);
@@ -1633,9 +1680,10 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
     }
 #undef TULA_UPD
     if (rc) return rc;
+    record(hp->trace_events[3], s);
     if (sw) rc = launch_combine<1>(n, numels, c2, sc, s);
     if (rc) return rc;
-    record(hp->trace_events[2], s);
+    record(hp->trace_events[4], s);
     return TULA_OK;
 }
 
@@ -1697,7 +1745,8 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
             dst[1] = g_large[p];
             dst[2] = hp->scale_elem[p];
         };
-        return launch_streaming<kNP3>(k_scale_elem, n, numels, 4096, 0, sc, hp->grid_ctas, s,
+        return launch_streaming<kNP3>(k_scale_elem, n, numels, 4096, kScaleThreads, 0, sc,
+                                      hp->grid_ctas, s,
                                       fill);
     }
     int rc = check_ws(hp->workspace, hp->workspace_bytes, n, pl);
@@ -1709,7 +1758,8 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
         dst[1] = nullptr;
         dst[2] = g_small[p];
     };
-    return run_reduce_k<1, false, false, true, true>(1, n, numels, sc, hp->grid_ctas, s, fill);
+    return run_reduce_k<1, false, false, true, true>(1, n, numels, sc, hp->grid_ctas, s, fill,
+                                                     nullptr);
 }
 
 const char *tula_ags_error_string(int code) {

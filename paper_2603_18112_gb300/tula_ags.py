@@ -52,7 +52,7 @@ class tula_ags_hparams(ctypes.Structure):
         ("lars_trust", c_float),
         ("scale", c_void_p), ("scale_elem", c_void_p), ("state", c_void_p),
         ("layer_stats", c_void_p), ("workspace", c_void_p), ("workspace_bytes", c_size_t),
-        ("grid_ctas", c_int), ("trace_events", c_void_p * 3),
+        ("grid_ctas", c_int), ("trace_events", c_void_p * 5),
     ]
 
 
@@ -85,7 +85,7 @@ def lib() -> ctypes.CDLL:
     L.tula_ags_last_cuda_error.restype = c_int
     L.tula_ags_launch_count.restype = ctypes.c_uint64
     L.tula_ags_plan_chunks.argtypes = [i64p, c_int, c_int, i64p]
-    L.tula_ags_chunk_elems.argtypes = [c_int]
+    L.tula_ags_chunk_elems.argtypes = [c_int, c_int]
     L.tula_ags_chunk_elems.restype = c_int
     L.tula_ags_workspace_error.argtypes = [c_void_p, c_size_t, i64p, c_int, c_int,
                                            ctypes.POINTER(c_int)]
@@ -158,8 +158,9 @@ def tula_ags_launch_count() -> int:
     return lib().tula_ags_launch_count()
 
 
-def tula_ags_chunk_elems(streams: int) -> int:
-    return lib().tula_ags_chunk_elems(streams)
+def tula_ags_chunk_elems(pass_: int, streams: int) -> int:
+    """Elements per tile of pass 1 (reduction) or pass 2 (update) with `streams` streams."""
+    return lib().tula_ags_chunk_elems(pass_, streams)
 
 
 def tula_ags_workspace_error(workspace: torch.Tensor, numels, K: int) -> int:
@@ -302,9 +303,11 @@ class AGSOptimizerStep:
         torch.cuda.synchronize(dev)
 
     def set_trace_events(self, events):
-        """cudaEvent_t handles (or None) recorded before pass 1, between passes, after pass 2."""
-        for i in range(3):
-            ev = events[i] if events is not None else None
+        """Up to five cudaEvent_t handles (or None) recorded at the kernel boundaries of a
+        step: before the reduction, after it, after its combine, after the update, after the
+        update's combine."""
+        for i in range(5):
+            ev = events[i] if events is not None and i < len(events) else None
             self.hp.trace_events[i] = (ev.cuda_event if hasattr(ev, "cuda_event") else ev) or None
 
     def error(self) -> int:

@@ -39,21 +39,23 @@ def test_defaults_match_paper(lib):
         assert not hp.scale and not hp.state and not hp.workspace
 
 
-@pytest.mark.parametrize("streams", [1, 2, 3, 4, 9, 17, 18])
-def test_tile_fits_one_stage(lib, streams):
-    C = T.tula_ags_chunk_elems(streams)
-    assert C % 128 == 0 and 0 < C * 4 * streams <= 32 * 1024
-    assert C * 4 * streams > 32 * 1024 - 128 * 4 * streams  # the largest multiple of 128 that fits
+@pytest.mark.parametrize("pass_,stage_kb,streams", [(1, 32, s) for s in (1, 2, 3, 4, 9, 17, 18)]
+                         + [(2, 24, s) for s in (2, 3, 4)])
+def test_tile_fits_one_stage(lib, pass_, stage_kb, streams):
+    C = T.tula_ags_chunk_elems(pass_, streams)
+    stage = stage_kb * 1024
+    assert C % 128 == 0 and 0 < C * 4 * streams <= stage
+    assert C * 4 * streams > stage - 128 * 4 * streams  # the largest multiple of 128 that fits
 
 
-def test_tile_sizes_reject_bad_stream_counts(lib):
-    assert T.lib().tula_ags_chunk_elems(0) == T.TULA_ERR_ARG
-    assert T.lib().tula_ags_chunk_elems(19) == T.TULA_ERR_ARG
+def test_tile_sizes_reject_bad_arguments(lib):
+    for pass_, streams in ((1, 0), (1, 19), (2, 0), (2, 5), (0, 2), (3, 2)):
+        assert T.lib().tula_ags_chunk_elems(pass_, streams) == T.TULA_ERR_ARG
 
 
 @pytest.mark.parametrize("streams", [1, 9])
 def test_plan_covers_every_element_once(lib, streams):
-    C = T.tula_ags_chunk_elems(streams)
+    C = T.tula_ags_chunk_elems(1, streams)
     numels = [0, 1, 3, C - 1, C, C + 1, 5 * C + 7, 64]
     starts = T.tula_ags_plan_chunks(numels, C)
     assert starts[0] == 0
@@ -85,7 +87,7 @@ def test_workspace_size_rejects(lib, numels, K):
 def test_per_tensor_size_limit(lib, K):
     """One tensor may span at most 6618 combine segments of 256 tiles (the
     header's stated limit); the check happens before any launch."""
-    tile = min(T.tula_ags_chunk_elems(K + 2 if K == 1 else K + 1), T.tula_ags_chunk_elems(4))
+    tile = min(T.tula_ags_chunk_elems(1, K + 2 if K == 1 else K + 1), T.tula_ags_chunk_elems(2, 4))
     limit = 1_694_208 * tile
     assert T.tula_ags_workspace_size([limit], K) > 0
     with pytest.raises(T.TulaError) as e:
