@@ -57,6 +57,23 @@ def _dist():
     return ws, rank, local
 
 
+def max_over_ranks(ms: float, device="cuda") -> float:
+    """The job's time: the slowest rank's (every rank calls this; one process: unchanged)."""
+    import torch
+    import torch.distributed as dist
+    if not dist.is_initialized() or dist.get_world_size() == 1:
+        return ms
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(params_per_rank: int, steps: int, world_size: int, t_max_ms: float) -> float:
+    """Parameters updated per second by the whole job: every rank runs its own replica of the
+    step (weak scaling), and the job takes as long as its slowest rank."""
+    return world_size * params_per_rank * steps / (t_max_ms / 1e3)
+
+
 # ---------------------------------------------------------------------------
 # bytes per parameter (fp32)
 # ---------------------------------------------------------------------------
@@ -357,11 +374,7 @@ def run_ours(args, wl):
     t_upd = [e[2].elapsed_time(e[3]) for e in evs]
     t_cmb2 = [e[3].elapsed_time(e[4]) for e in evs]
 
-    t_max_ms = elapsed_ms
-    if ws > 1:
-        tt = torch.tensor([elapsed_ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        t_max_ms = float(tt.item())
+    t_max_ms = max_over_ranks(elapsed_ms)
 
     # ---- end to end through the C ABI with host buffers -------------------
     e2e = None
@@ -387,12 +400,8 @@ def run_ours(args, wl):
             host_stats.copy_(step.stats, non_blocking=True)
         e_end.record(stream)
     stream.synchronize()
-    e2e_ms = e_start.elapsed_time(e_end)
-    if ws > 1:
-        tt = torch.tensor([e2e_ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
-    e2e = {"value": ws * N * args.e2e_steps / (e2e_ms / 1e3), "unit": UNIT,
+    e2e_ms = max_over_ranks(e_start.elapsed_time(e_end))
+    e2e = {"value": job_throughput(N, args.e2e_steps, ws, e2e_ms), "unit": UNIT,
            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": args.e2e_steps}
 
     if rank != 0:
@@ -409,7 +418,7 @@ def run_ours(args, wl):
     step_gbs = step_min_bytes_per_param(K) * N / (ms_per_step / 1e3) / 1e9
     traffic = _ncu_traffic("k_reduce", wl.name, N)
     line = {
-        "metric": METRIC, "value": ws * N * args.steps / (t_max_ms / 1e3), "unit": UNIT,
+        "metric": METRIC, "value": job_throughput(N, args.steps, ws, t_max_ms), "unit": UNIT,
         "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
         "steps_per_s": 1e3 / ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic",
