@@ -75,8 +75,9 @@ struct Ring {
 // consumers, not HBM, set the pace with three warps, so it runs four.
 using Ring1 = Ring<32, 6, 3>;
 using Ring2 = Ring<24, 8, 4>;
-constexpr int kDynTiles = 128;           // tiles per CTA from which a launch claims its tiles
+constexpr int kDynTiles = 64;            // tiles per CTA from which a launch claims its tiles
 constexpr unsigned kClaim = 4;           // tiles per claim
+constexpr unsigned kClaimTail = 8;       // single-tile claims for the last kClaimTail per CTA
 constexpr int kPend = 4;                // tiles whose warp reductions run together
 constexpr int kCombWarps = 4;           // k_combine: one warp per segment, 4 per CTA
 constexpr int kSegTiles = 256;          // tile partials per combine segment (8 per lane)
@@ -125,12 +126,13 @@ struct CombTable {
 
 struct Scalars {
     int K, rule, gran, force, refresh, mode, n_total, read_w;
-    int pow2K, evict_first, pad1, pad2;  // evict_first: TMA loads ask L2 to drop their lines first
+    int pow2K, evict_first, n_seg1, pad2;  // evict_first: TMA loads ask L2 to drop their lines
+                                           // first; n_seg1: combine segments of pass 1
     float delta, eps, s_max, static_s, lars_trust, lr, mu, wd, invK, Kf;
     float *scale;
     double *state;
     double *stats;
-    unsigned *done;  // [0]: tensors combined after pass 1
+    unsigned *done;  // [1]: segments combined in a step (the branch's ticket)
     int *flags;      // [0]: branch of the last step (1 = scaled)
     unsigned *err;   // [0]: bounded waits that ran out (sticky until read)
     unsigned *sctr1; // [tensor]: segments combined, pass 1
@@ -407,8 +409,9 @@ struct TensorCache {
 //  * round-robin (tile blockIdx.x + j * gridDim.x), for launches of fewer than
 //    kDynTiles tiles per CTA: nothing to claim, nothing to wait for;
 //  * claimed, for larger launches: the producer warp of each CTA takes kClaim
-//    consecutive tiles at a time from a global counter (ctr[0]), two claims
-//    ahead to hide the atomic's latency.  SMs do not stream at equal rates (on
+//    consecutive tiles at a time from a global counter (ctr[0]), with one
+//    claim in flight while it issues the range before (see produce()).  SMs
+//    do not stream at equal rates (on
 //    large launches the last CTA of a round-robin deal finished 15-30% after
 //    the median), so claiming lets the faster SMs take more tiles and the
 //    launch end with the memory system rather than with its slowest SM.  The
@@ -423,7 +426,9 @@ struct TensorCache {
 // offset i * chunk floats of the stage.  With `reverse` the order is mirrored
 // (pass 2 walks the tiles backwards, so it starts on what pass 1 left in L2).
 
-__device__ __forceinline__ unsigned claim_tiles(unsigned *ctr) { return atomicAdd(ctr, 1u); }
+__device__ __forceinline__ unsigned claim_tiles(unsigned *ctr, unsigned n) {
+    return atomicAdd(ctr, n);
+}
 
 // Round-robin tiles of this CTA (0 when the launch claims its tiles).
 __device__ __forceinline__ int static_tiles(int nc) {
@@ -449,11 +454,17 @@ __device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
     const bool hint = sc.evict_first != 0;
     const uint64_t policy = policy_evict_first();
     TensorCache tc;
-    unsigned next0 = 0u, next1 = 0u, used = 0u;  // claims in flight, tiles used of next0
-    if (claim && lane == 0) {
-        next0 = claim_tiles(ctr);
-        next1 = claim_tiles(ctr);
-    }
+    // Claiming (lane 0): tiles [cur, cur_end) are being issued, [nxt, nxt_end) come next and
+    // one claim is in flight.  The first two ranges of each CTA are dealt, not claimed (152
+    // CTAs claiming at once would queue on the counter at the start); claimed ranges begin
+    // after them.  Near the end, claims shrink to one tile so that CTAs do not hold tiles
+    // others could have taken.
+    const unsigned G = gridDim.x, b = blockIdx.x;
+    const unsigned base = 2u * G * kClaim;
+    unsigned cur = b * kClaim, cur_end = cur + kClaim;
+    unsigned nxt = (G + b) * kClaim, nxt_end = nxt + kClaim;
+    unsigned pend = 0u, pend_k = kClaim;
+    if (claim && lane == 0) pend = claim_tiles(ctr, kClaim);
     int issued = 0, ending = 0;
     for (int j = 0; ending < R::kConsumers; ++j) {
         const int s = j % R::kStages;
@@ -462,14 +473,19 @@ __device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
             i = blockIdx.x + (unsigned)j * gridDim.x;
         } else if (claim) {
             if (lane == 0) {
-                if (used == kClaim) {
-                    next0 = next1;
-                    used = 0u;
-                    // the counter only grows: no more claims once past the end
-                    if (next0 * kClaim < nc) next1 = claim_tiles(ctr);
+                if (cur == cur_end) {
+                    cur = nxt;
+                    cur_end = nxt_end;
+                    if (nxt < nc) {  // the counter only grows: no more claims once past the end
+                        nxt = base + pend;
+                        nxt_end = nxt + pend_k;
+                        if (nxt < nc) {
+                            pend_k = nxt + kClaimTail * G >= nc ? 1u : kClaim;
+                            pend = claim_tiles(ctr, pend_k);
+                        }
+                    }
                 }
-                i = next0 * kClaim + used;
-                ++used;
+                i = cur++;
             }
             i = __shfl_sync(kFull, i, 0);
         }
@@ -873,12 +889,12 @@ __device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, dou
 }
 
 // |G|^2, Delta (Eq. 5) and the branch of Algorithm 1 (one warp, after every
-// tensor's sums are in sc.tsum).
+// segment's |gbar|^2 is in sc.spart1; segments in index order, then a fixed tree).
 __device__ void finalize_step(const Scalars &sc) {
     const int lane = threadIdx.x & 31;
     double v[1] = {0.0};
-    for (int t = lane; t < sc.n_total; t += 32)
-        v[0] = __dadd_rn(v[0], __ldcg(&sc.tsum[(size_t)t * kTsum + 0]));
+    for (int g = lane; g < sc.n_seg1; g += 32)
+        v[0] = __dadd_rn(v[0], __ldcg(&sc.spart1[(size_t)g * kAcc + 0]));
     warp_sums<1>(v);
     if (lane != 0) return;
     const double g2 = v[0];
@@ -895,7 +911,7 @@ __device__ void finalize_step(const Scalars &sc) {
     sc.state[TULA_STATE_DELTA] = dv;
     sc.state[TULA_STATE_SCALED] = (double)scaled;
     sc.flags[0] = scaled;
-    sc.done[0] = 0u;  // re-arm for the next call
+    sc.done[1] = 0u;  // re-arm for the next call
 }
 
 template <int NA>
@@ -940,18 +956,32 @@ __global__ void __launch_bounds__(32 * kCombWarps)
     }
     warp_sums<NA>(v);
 
-    if (nseg > 1) {
-        // Hand the segment sum over; the warp taking the tensor's last ticket adds
-        // the segment sums in order.
-        int last = 0;
-        const long long sg0 = (long long)tab.s0 + tab.sfirst[t];
+    // The branch needs only |G|^2, so it does not wait for the tensors: in a step,
+    // every segment posts its sums and takes a ticket over all segments, and the
+    // warp taking the last one forms |G|^2, Delta and the branch while the
+    // tensors are being finished.  A tensor of several segments is finished by
+    // the warp taking its last segment ticket, which adds the segment sums in
+    // order.
+    const bool step = NA == kAcc && sc.mode == kModeStep;
+    const long long sg0 = (long long)tab.s0 + tab.sfirst[t];
+    int last_all = 0, last_seg = 1;
+    if (nseg > 1 || step) {
         if (lane == 0) {
 #pragma unroll
             for (int a = 0; a < NA; ++a) spart[(sg0 + k) * NA + a] = v[a];
             __threadfence();
-            last = atomicAdd(&sctr[tg], 1u) == (unsigned)(nseg - 1);
+            if (step) last_all = atomicAdd(&sc.done[1], 1u) == (unsigned)(sc.n_seg1 - 1);
+            if (nseg > 1) last_seg = atomicAdd(&sctr[tg], 1u) == (unsigned)(nseg - 1);
         }
-        if (!__shfl_sync(kFull, last, 0)) return;
+        last_all = __shfl_sync(kFull, last_all, 0);
+        last_seg = __shfl_sync(kFull, last_seg, 0);
+    }
+    if (last_all) {
+        __threadfence();
+        finalize_step(sc);
+    }
+    if (!last_seg) return;
+    if (nseg > 1) {
         __threadfence();
 #pragma unroll
         for (int a = 0; a < NA; ++a) v[a] = 0.0;
@@ -965,18 +995,7 @@ __global__ void __launch_bounds__(32 * kCombWarps)
 
     // This warp holds tensor tg's sums (lane 0).
     if constexpr (NA == kAcc) {
-        int last = 0;
         tensor_done(sc, tg, v[0], v[1], v[2], scale_old);
-        if (lane == 0) {
-            if (sc.mode == kModeStep) {
-                __threadfence();
-                last = atomicAdd(&sc.done[0], 1u) == (unsigned)(sc.n_total - 1);
-            }
-        }
-        if (__shfl_sync(kFull, last, 0)) {
-            __threadfence();
-            finalize_step(sc);
-        }
     } else {
         // lanes 0 and 1 take the two square roots in one instruction
         const double sw = __shfl_sync(kFull, v[0], 0);
@@ -1407,8 +1426,12 @@ int launch_streaming(Kernel kernel, int n, const int64_t *numels, int chunk, int
 
 // k_combine over all tensors (tiles of `chunk` elements), NA sums per tile.
 template <int NA>
-int launch_combine(int n, const int64_t *numels, int chunk, const Scalars &sc, cudaStream_t s) {
+int launch_combine(int n, const int64_t *numels, int chunk, const Scalars &sc_in, cudaStream_t s) {
     std::unique_ptr<CombTable> tab(new CombTable);
+    Scalars sc = sc_in;
+    long long segs_total = 0;  // the branch's ticket runs over every segment of every launch
+    for (int p = 0; p < n; ++p) segs_total += segs_of(tiles_of(numels[p], chunk));
+    sc.n_seg1 = (int)segs_total;
     long long c_global = 0, s_global = 0;
     int p = 0;
     while (p < n) {
