@@ -137,10 +137,10 @@ struct Scalars {
     unsigned *err;   // [0]: bounded waits that ran out (sticky until read)
     unsigned *sctr1; // [tensor]: segments combined, pass 1
     unsigned *sctr2; // [tensor]: segments combined, pass 2
-    double *part1;   // [tile][kAcc], pass 1
-    double *part2;   // [tile], pass 2 (|w|^2)
-    double *spart1;  // [segment][kAcc], pass 1
-    double *spart2;  // [segment], pass 2
+    float2 *part1;   // [tile][kAcc], pass 1 (float-float sums)
+    float2 *part2;   // [tile], pass 2 (|w|^2)
+    float2 *spart1;  // [segment][kAcc], pass 1
+    float2 *spart2;  // [segment], pass 2
     double *tsum;    // [tensor][kTsum]: |gbar|^2, |g_0|^2, |w|^2
     float *cand;     // [tensor]: c_p of the scaled branch (AGS: the old gradscale)
     unsigned *tiles; // [2 * pass]: next tile to claim, [2 * pass + 1]: CTAs finished
@@ -232,6 +232,48 @@ __device__ __forceinline__ void warp_sums(float (&v)[R]) {
     }
 }
 
+// Float-float numbers (hi, lo as a float2, value hi + lo, |lo| <= ulp(hi) / 2)
+// carry the partial sums between kernels: they hold ~48 significant bits and
+// add on the FP32 pipes, where an fp64 add costs ~64x more on this part.
+// Knuth's TwoSum: s + e == a + b exactly.
+__device__ __forceinline__ float2 two_sum(float a, float b) {
+    const float s = __fadd_rn(a, b);
+    const float bb = __fsub_rn(s, a);
+    const float e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+    return make_float2(s, e);
+}
+// a + b for float-float a, b: TwoSum of the high parts, the low parts added to
+// the error, then Dekker's Fast2Sum to renormalise.  All terms here are sums of
+// squares (no cancellation): relative error below 2^-46 per addition.
+__device__ __forceinline__ float2 ff_add(float2 a, float2 b) {
+    const float2 s = two_sum(a.x, b.x);
+    const float e = __fadd_rn(s.y, __fadd_rn(a.y, b.y));
+    const float hi = __fadd_rn(s.x, e);
+    return make_float2(hi, __fsub_rn(e, __fsub_rn(hi, s.x)));
+}
+__device__ __forceinline__ float2 ff_from_double(double d) {
+    const float hi = __double2float_rn(d);
+    return make_float2(hi, __double2float_rn(__dsub_rn(d, (double)hi)));
+}
+__device__ __forceinline__ double ff_to_double(float2 v) {
+    return __dadd_rn((double)v.x, (double)v.y);
+}
+// Fixed-tree warp sum of R float-float values (lane 0 gets the sums).
+template <int R>
+__device__ __forceinline__ void warp_sums_ff(float2 (&v)[R]) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        float2 t[R];
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            t[r].x = __shfl_down_sync(kFull, v[r].x, o);
+            t[r].y = __shfl_down_sync(kFull, v[r].y, o);
+        }
+#pragma unroll
+        for (int r = 0; r < R; ++r) v[r] = ff_add(v[r], t[r]);
+    }
+}
+
 // ----------------------------------------------------------------------------
 // Device helpers: programmatic dependent launch, mbarrier, TMA (inline PTX)
 // ----------------------------------------------------------------------------
@@ -312,6 +354,15 @@ __device__ __forceinline__ uint64_t policy_evict_first() {
     asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
     return p;
 }
+
+// Ticket counter increment with acquire-release semantics at GPU scope: the
+// caller's earlier stores are visible to whoever later takes the last ticket.
+__device__ __forceinline__ unsigned ticket(unsigned *ctr) {
+    unsigned r;
+    asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], 1;" : "=r"(r) : "l"(ctr) : "memory");
+    return r;
+}
+__device__ __forceinline__ void fence_acq_rel() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
 
 __device__ __forceinline__ void report_timeout(const Scalars &sc) {
     atomicOr(sc.err, 1u);
@@ -799,11 +850,11 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
 #pragma unroll
             for (int p = 0; p < kPend; ++p)
                 if (ptile[p] >= 0) {
-                    double *P = sc.part1 + (size_t)ptile[p] * kAcc;
+                    float2 *P = sc.part1 + (size_t)ptile[p] * kAcc;
 #pragma unroll
                     for (int a = 0; a < kAcc; ++a) {
-                        if constexpr (PR) P[a] = pendd[p * kAcc + a];
-                        else P[a] = (double)pendf[p * kAcc + a];
+                        if constexpr (PR) P[a] = ff_from_double(pendd[p * kAcc + a]);
+                        else P[a] = make_float2(pendf[p * kAcc + a], 0.f);
                     }
                 }
         }
@@ -890,16 +941,14 @@ __device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, dou
 
 // |G|^2, Delta (Eq. 5) and the branch of Algorithm 1 (one warp, after every
 // segment's |gbar|^2 is in sc.spart1; segments in index order, then a fixed tree).
-__device__ void finalize_step(const Scalars &sc) {
+__device__ void finalize_step(const Scalars &sc, double g2_prev, double steps) {
     const int lane = threadIdx.x & 31;
-    double v[1] = {0.0};
+    float2 v[1] = {make_float2(0.f, 0.f)};
     for (int g = lane; g < sc.n_seg1; g += 32)
-        v[0] = __dadd_rn(v[0], __ldcg(&sc.spart1[(size_t)g * kAcc + 0]));
-    warp_sums<1>(v);
+        v[0] = ff_add(v[0], __ldcg(&sc.spart1[(size_t)g * kAcc + 0]));
+    warp_sums_ff<1>(v);
     if (lane != 0) return;
-    const double g2 = v[0];
-    const double g2_prev = sc.state[TULA_STATE_G2_PREV];
-    const double steps = sc.state[TULA_STATE_STEPS];
+    const double g2 = ff_to_double(v[0]);
     // no previous step -> +inf (sensitive)
     const double dv = steps == 0.0 ? (double)INFINITY : fabs((g2 - g2_prev) / g2_prev);
     int scaled;
@@ -917,30 +966,37 @@ __device__ void finalize_step(const Scalars &sc) {
 template <int NA>
 __global__ void __launch_bounds__(32 * kCombWarps)
     k_combine(const __grid_constant__ CombTable tab, const __grid_constant__ Scalars sc) {
-    grid_dependency();
+    // Everything that does not come from the kernel before is read ahead of the
+    // wait for it (this kernel is launched early and waits through most of the
+    // previous one): the segment's place in the table and, in a step, the old
+    // gradscale and the step record, which earlier kernels wrote.
     const int lane = threadIdx.x & 31;
     const int seg = (int)blockIdx.x * kCombWarps + (int)(threadIdx.x >> 5);
-    if (seg >= tab.ns) return;
-    const int t = tab.seg_t[seg];
+    const bool active = seg < tab.ns;
+    const int t = active ? tab.seg_t[seg] : 0;
     const int tg = tab.t0 + t;
-    // gradscale of this tensor, needed by the epilogue: load it now (AGS step)
-    const float scale_old = (NA == kAcc && sc.mode == kModeStep && sc.scale) ? sc.scale[tg] : 1.0f;
     const int k = seg - tab.sfirst[t];                 // segment within the tensor
     const int nseg = tab.sfirst[t + 1] - tab.sfirst[t];
-    const double *part = NA == kAcc ? sc.part1 : sc.part2;
-    double *spart = NA == kAcc ? sc.spart1 : sc.spart2;
-    unsigned *sctr = NA == kAcc ? sc.sctr1 : sc.sctr2;
     const long long first = (long long)tab.cfirst[t] + (long long)k * kSegTiles;
     const int n = min(kSegTiles, tab.ntiles[t] - k * kSegTiles);
+    const bool step = NA == kAcc && sc.mode == kModeStep;
+    const float scale_old = (active && step && sc.scale) ? sc.scale[tg] : 1.0f;
+    const double g2_prev = step ? sc.state[TULA_STATE_G2_PREV] : 0.0;
+    const double steps = step ? sc.state[TULA_STATE_STEPS] : 0.0;
+    grid_dependency();
+    if (!active) return;
+    const float2 *part = NA == kAcc ? sc.part1 : sc.part2;
+    float2 *spart = NA == kAcc ? sc.spart1 : sc.spart2;
+    unsigned *sctr = NA == kAcc ? sc.sctr1 : sc.sctr2;
 
     // The segment's tiles: lane i adds tiles i, i + 32, ... in order (8 loads in
     // flight), then a fixed tree across the warp.
-    double v[NA];
+    float2 v[NA];
 #pragma unroll
-    for (int a = 0; a < NA; ++a) v[a] = 0.0;
+    for (int a = 0; a < NA; ++a) v[a] = make_float2(0.f, 0.f);
     int i = lane;
     for (; i + 7 * 32 < n; i += 8 * 32) {
-        double x[8][NA];
+        float2 x[8][NA];
 #pragma unroll
         for (int u = 0; u < 8; ++u)
 #pragma unroll
@@ -948,13 +1004,13 @@ __global__ void __launch_bounds__(32 * kCombWarps)
 #pragma unroll
         for (int u = 0; u < 8; ++u)
 #pragma unroll
-            for (int a = 0; a < NA; ++a) v[a] = __dadd_rn(v[a], x[u][a]);
+            for (int a = 0; a < NA; ++a) v[a] = ff_add(v[a], x[u][a]);
     }
     for (; i < n; i += 32) {
 #pragma unroll
-        for (int a = 0; a < NA; ++a) v[a] = __dadd_rn(v[a], part[(first + i) * NA + a]);
+        for (int a = 0; a < NA; ++a) v[a] = ff_add(v[a], part[(first + i) * NA + a]);
     }
-    warp_sums<NA>(v);
+    warp_sums_ff<NA>(v);
 
     // The branch needs only |G|^2, so it does not wait for the tensors: in a step,
     // every segment posts its sums and takes a ticket over all segments, and the
@@ -962,43 +1018,43 @@ __global__ void __launch_bounds__(32 * kCombWarps)
     // tensors are being finished.  A tensor of several segments is finished by
     // the warp taking its last segment ticket, which adds the segment sums in
     // order.
-    const bool step = NA == kAcc && sc.mode == kModeStep;
     const long long sg0 = (long long)tab.s0 + tab.sfirst[t];
     int last_all = 0, last_seg = 1;
     if (nseg > 1 || step) {
         if (lane == 0) {
 #pragma unroll
             for (int a = 0; a < NA; ++a) spart[(sg0 + k) * NA + a] = v[a];
-            __threadfence();
-            if (step) last_all = atomicAdd(&sc.done[1], 1u) == (unsigned)(sc.n_seg1 - 1);
-            if (nseg > 1) last_seg = atomicAdd(&sctr[tg], 1u) == (unsigned)(nseg - 1);
+            // the tickets release the stores above; the warp taking a last one acquires
+            if (step) last_all = ticket(&sc.done[1]) == (unsigned)(sc.n_seg1 - 1);
+            if (nseg > 1) last_seg = ticket(&sctr[tg]) == (unsigned)(nseg - 1);
         }
         last_all = __shfl_sync(kFull, last_all, 0);
         last_seg = __shfl_sync(kFull, last_seg, 0);
     }
     if (last_all) {
-        __threadfence();
-        finalize_step(sc);
+        fence_acq_rel();
+        finalize_step(sc, g2_prev, steps);
     }
     if (!last_seg) return;
     if (nseg > 1) {
-        __threadfence();
+        fence_acq_rel();
 #pragma unroll
-        for (int a = 0; a < NA; ++a) v[a] = 0.0;
+        for (int a = 0; a < NA; ++a) v[a] = make_float2(0.f, 0.f);
         for (int j = lane; j < nseg; j += 32) {
 #pragma unroll
-            for (int a = 0; a < NA; ++a) v[a] = __dadd_rn(v[a], __ldcg(&spart[(sg0 + j) * NA + a]));
+            for (int a = 0; a < NA; ++a) v[a] = ff_add(v[a], __ldcg(&spart[(sg0 + j) * NA + a]));
         }
-        warp_sums<NA>(v);
+        warp_sums_ff<NA>(v);
         if (lane == 0) sctr[tg] = 0u;  // re-arm
     }
 
     // This warp holds tensor tg's sums (lane 0).
     if constexpr (NA == kAcc) {
-        tensor_done(sc, tg, v[0], v[1], v[2], scale_old);
+        tensor_done(sc, tg, ff_to_double(v[0]), ff_to_double(v[1]), ff_to_double(v[2]),
+                    scale_old);
     } else {
         // lanes 0 and 1 take the two square roots in one instruction
-        const double sw = __shfl_sync(kFull, v[0], 0);
+        const double sw = __shfl_sync(kFull, ff_to_double(v[0]), 0);
         const double sg = sc.tsum[(size_t)tg * kTsum + 0];
         const double r = sqrt(lane == 0 ? sw : sg);
         const double nw = __shfl_sync(kFull, r, 0), ng = __shfl_sync(kFull, r, 1);
@@ -1185,7 +1241,7 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
             if (lane == 0) {
 #pragma unroll
                 for (int p = 0; p < kPend; ++p)
-                    if (ptile[p] >= 0) sc.part2[ptile[p]] = (double)pend[p];
+                    if (ptile[p] >= 0) sc.part2[ptile[p]] = make_float2(pend[p], 0.f);
             }
         }
         if (stop) break;
@@ -1279,10 +1335,10 @@ WsLayout ws_layout(int n_tensors, const Plan &pl) {
     L.tiles = take(sizeof(unsigned) * 4);
     L.sctr1 = take(sizeof(unsigned) * (size_t)n_tensors);
     L.sctr2 = take(sizeof(unsigned) * (size_t)n_tensors);
-    L.part1 = take(sizeof(double) * kAcc * (size_t)pl.c1);
-    L.part2 = take(sizeof(double) * (size_t)pl.c2);
-    L.spart1 = take(sizeof(double) * kAcc * (size_t)pl.s1);
-    L.spart2 = take(sizeof(double) * (size_t)pl.s2);
+    L.part1 = take(sizeof(float2) * kAcc * (size_t)pl.c1);
+    L.part2 = take(sizeof(float2) * (size_t)pl.c2);
+    L.spart1 = take(sizeof(float2) * kAcc * (size_t)pl.s1);
+    L.spart2 = take(sizeof(float2) * (size_t)pl.s2);
     L.tsum = take(sizeof(double) * kTsum * (size_t)n_tensors);
     L.cand = take(sizeof(float) * (size_t)n_tensors);
     L.total = off;
@@ -1495,10 +1551,10 @@ Scalars make_scalars(const tula_ags_hparams *hp, int K, int n, void *ws, const W
     sc.tiles = reinterpret_cast<unsigned *>(b + L.tiles);
     sc.sctr1 = reinterpret_cast<unsigned *>(b + L.sctr1);
     sc.sctr2 = reinterpret_cast<unsigned *>(b + L.sctr2);
-    sc.part1 = reinterpret_cast<double *>(b + L.part1);
-    sc.part2 = reinterpret_cast<double *>(b + L.part2);
-    sc.spart1 = reinterpret_cast<double *>(b + L.spart1);
-    sc.spart2 = reinterpret_cast<double *>(b + L.spart2);
+    sc.part1 = reinterpret_cast<float2 *>(b + L.part1);
+    sc.part2 = reinterpret_cast<float2 *>(b + L.part2);
+    sc.spart1 = reinterpret_cast<float2 *>(b + L.spart1);
+    sc.spart2 = reinterpret_cast<float2 *>(b + L.spart2);
     sc.tsum = reinterpret_cast<double *>(b + L.tsum);
     sc.cand = reinterpret_cast<float *>(b + L.cand);
     return sc;
