@@ -777,7 +777,14 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
     constexpr int KS = P1<KT>::KS;
     constexpr int NSMAX = KS + 2;
     extern __shared__ __align__(128) unsigned char smem[];
-    grid_dependency();
+    // In a step that does not read w, the kernels still running before this one
+    // (the previous step's update and combine) write nothing this kernel loads:
+    // the producer of the pass's first launch streams replicas in right away,
+    // and only the consumers, which write the mean over replica 0 and the tile
+    // partials, wait for them.  Otherwise the whole CTA waits first.
+    grid_launch_dependents();
+    const bool early = !RW && !SS && sc.mode == kModeStep && tab.first;
+    if (!early) grid_wait();
     uint64_t *full, *empty;
     int *stage_tile;
     ring_setup<Ring1>(smem, full, empty, stage_tile);
@@ -797,6 +804,7 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
                                    empty, stage_tile);
         return;
     }
+    if (early) grid_wait();
     const int my_role = lane < ns ? roles[lane] : 0;
 
     const int cw = warp - 1;
