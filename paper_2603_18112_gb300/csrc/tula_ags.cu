@@ -77,7 +77,7 @@ using Ring1 = Ring<32, 6, 3>;
 using Ring2 = Ring<24, 8, 4>;
 constexpr int kDynTiles = 64;            // tiles per CTA from which a launch claims its tiles
 constexpr unsigned kClaim = 4;           // tiles per claim
-constexpr unsigned kClaimTail = 8;       // single-tile claims for the last kClaimTail per CTA
+constexpr unsigned kClaimTail = 16;      // single-tile claims for the last kClaimTail per CTA
 constexpr int kPend = 4;                // tiles whose warp reductions run together
 constexpr int kCombWarps = 4;           // k_combine: one warp per segment, 4 per CTA
 constexpr int kSegTiles = 256;          // tile partials per combine segment (8 per lane)
@@ -155,6 +155,18 @@ __device__ __forceinline__ void st_stream(float *p, float4 v) {
 }
 __device__ __forceinline__ void st_keep(float *p, float4 v) {
     *reinterpret_cast<float4 *>(p) = v;
+}
+// 8-byte store that asks L2 to keep the line: tile partials, read back by the
+// combine kernel right after the streaming kernel that writes them.
+__device__ __forceinline__ void st_keep_l2(float2 *p, float2 v, uint64_t policy) {
+    asm volatile("st.global.L2::cache_hint.v2.f32 [%0], {%1, %2}, %3;" ::"l"(p), "f"(v.x), "f"(v.y),
+                 "l"(policy)
+                 : "memory");
+}
+__device__ __forceinline__ uint64_t policy_evict_last() {
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
 }
 // 16-byte load from shared memory (a shared-window address).
 __device__ __forceinline__ float4 lds4(uint32_t addr) {
@@ -859,10 +871,11 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
             for (int p = 0; p < kPend; ++p)
                 if (ptile[p] >= 0) {
                     float2 *P = sc.part1 + (size_t)ptile[p] * kAcc;
+                    const uint64_t keep = policy_evict_last();
 #pragma unroll
                     for (int a = 0; a < kAcc; ++a) {
-                        if constexpr (PR) P[a] = ff_from_double(pendd[p * kAcc + a]);
-                        else P[a] = make_float2(pendf[p * kAcc + a], 0.f);
+                        if constexpr (PR) st_keep_l2(P + a, ff_from_double(pendd[p * kAcc + a]), keep);
+                        else st_keep_l2(P + a, make_float2(pendf[p * kAcc + a], 0.f), keep);
                     }
                 }
         }
@@ -952,8 +965,16 @@ __device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, dou
 __device__ void finalize_step(const Scalars &sc, double g2_prev, double steps) {
     const int lane = threadIdx.x & 31;
     float2 v[1] = {make_float2(0.f, 0.f)};
-    for (int g = lane; g < sc.n_seg1; g += 32)
-        v[0] = ff_add(v[0], __ldcg(&sc.spart1[(size_t)g * kAcc + 0]));
+    for (int g0 = 0; g0 < sc.n_seg1; g0 += 8 * 32) {  // 8 loads in flight per lane
+        float2 x[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int g = g0 + lane + 32 * u;
+            x[u] = g < sc.n_seg1 ? __ldcg(&sc.spart1[(size_t)g * kAcc + 0]) : make_float2(0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) v[0] = ff_add(v[0], x[u]);
+    }
     warp_sums_ff<1>(v);
     if (lane != 0) return;
     const double g2 = ff_to_double(v[0]);
@@ -1249,7 +1270,9 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
             if (lane == 0) {
 #pragma unroll
                 for (int p = 0; p < kPend; ++p)
-                    if (ptile[p] >= 0) sc.part2[ptile[p]] = make_float2(pend[p], 0.f);
+                    if (ptile[p] >= 0)
+                        st_keep_l2(sc.part2 + ptile[p], make_float2(pend[p], 0.f),
+                                   policy_evict_last());
             }
         }
         if (stop) break;
