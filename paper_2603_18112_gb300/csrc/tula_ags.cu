@@ -163,6 +163,9 @@ __device__ __forceinline__ void st_keep_l2(float2 *p, float2 v, uint64_t policy)
                  "l"(policy)
                  : "memory");
 }
+__device__ __forceinline__ void st_keep_l2(double *p, double v, uint64_t policy) {
+    asm volatile("st.global.L2::cache_hint.f64 [%0], %1, %2;" ::"l"(p), "d"(v), "l"(policy) : "memory");
+}
 __device__ __forceinline__ uint64_t policy_evict_last() {
     uint64_t p;
     asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
@@ -187,6 +190,8 @@ __device__ __forceinline__ float sq4(float acc, float4 v) {
 }
 
 // fp64 sum of exact squares (an fp32 square is exact in fp64), one DFMA per term
+// Precise sum of squares: each square is exact in fp64 and rounded once into
+// the running sum (this path is bound by GB300's FP64 throughput, not latency).
 __device__ __forceinline__ double dsq4(double acc, float4 v) {
     acc = __fma_rn((double)v.x, (double)v.x, acc);
     acc = __fma_rn((double)v.y, (double)v.y, acc);
@@ -263,14 +268,33 @@ __device__ __forceinline__ float2 ff_add(float2 a, float2 b) {
     const float hi = __fadd_rn(s.x, e);
     return make_float2(hi, __fsub_rn(e, __fsub_rn(hi, s.x)));
 }
-__device__ __forceinline__ float2 ff_from_double(double d) {
-    const float hi = __double2float_rn(d);
-    return make_float2(hi, __double2float_rn(__dsub_rn(d, (double)hi)));
-}
 __device__ __forceinline__ double ff_to_double(float2 v) {
     return __dadd_rn((double)v.x, (double)v.y);
 }
+// Partial sums travel as float-float pairs, or as fp64 where the norms feed a
+// coefficient (precise mode): Part<P>::T is the stored type, zero/add/tree work
+// on it.  Both are 8 bytes, so the workspace layout is the same.
+template <bool P>
+struct Part;
+template <>
+struct Part<false> {
+    using T = float2;
+    static __device__ __forceinline__ T zero() { return make_float2(0.f, 0.f); }
+    static __device__ __forceinline__ T add(T a, T b) { return ff_add(a, b); }
+    static __device__ __forceinline__ double value(T a) { return ff_to_double(a); }
+};
+template <>
+struct Part<true> {
+    using T = double;
+    static __device__ __forceinline__ T zero() { return 0.0; }
+    static __device__ __forceinline__ T add(T a, T b) { return __dadd_rn(a, b); }
+    static __device__ __forceinline__ double value(T a) { return a; }
+};
 // Fixed-tree warp sum of R float-float values (lane 0 gets the sums).
+template <int R>
+__device__ __forceinline__ void warp_sums_ff(double (&v)[R]) {
+    warp_sums<R>(v);
+}
 template <int R>
 __device__ __forceinline__ void warp_sums_ff(float2 (&v)[R]) {
 #pragma unroll
@@ -874,7 +898,7 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
                     const uint64_t keep = policy_evict_last();
 #pragma unroll
                     for (int a = 0; a < kAcc; ++a) {
-                        if constexpr (PR) st_keep_l2(P + a, ff_from_double(pendd[p * kAcc + a]), keep);
+                        if constexpr (PR) st_keep_l2(reinterpret_cast<double *>(P) + a, pendd[p * kAcc + a], keep);
                         else st_keep_l2(P + a, make_float2(pendf[p * kAcc + a], 0.f), keep);
                     }
                 }
@@ -962,22 +986,26 @@ __device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, dou
 
 // |G|^2, Delta (Eq. 5) and the branch of Algorithm 1 (one warp, after every
 // segment's |gbar|^2 is in sc.spart1; segments in index order, then a fixed tree).
+template <bool PREC>
 __device__ void finalize_step(const Scalars &sc, double g2_prev, double steps) {
+    using PT = Part<PREC>;
+    using T = typename PT::T;
+    const T *spart = reinterpret_cast<const T *>(sc.spart1);
     const int lane = threadIdx.x & 31;
-    float2 v[1] = {make_float2(0.f, 0.f)};
+    T v[1] = {PT::zero()};
     for (int g0 = 0; g0 < sc.n_seg1; g0 += 8 * 32) {  // 8 loads in flight per lane
-        float2 x[8];
+        T x[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
             const int g = g0 + lane + 32 * u;
-            x[u] = g < sc.n_seg1 ? __ldcg(&sc.spart1[(size_t)g * kAcc + 0]) : make_float2(0.f, 0.f);
+            x[u] = g < sc.n_seg1 ? __ldcg(&spart[(size_t)g * kAcc + 0]) : PT::zero();
         }
 #pragma unroll
-        for (int u = 0; u < 8; ++u) v[0] = ff_add(v[0], x[u]);
+        for (int u = 0; u < 8; ++u) v[0] = PT::add(v[0], x[u]);
     }
     warp_sums_ff<1>(v);
     if (lane != 0) return;
-    const double g2 = ff_to_double(v[0]);
+    const double g2 = PT::value(v[0]);
     // no previous step -> +inf (sensitive)
     const double dv = steps == 0.0 ? (double)INFINITY : fabs((g2 - g2_prev) / g2_prev);
     int scaled;
@@ -992,9 +1020,11 @@ __device__ void finalize_step(const Scalars &sc, double g2_prev, double steps) {
     sc.done[1] = 0u;  // re-arm for the next call
 }
 
-template <int NA>
+template <int NA, bool PREC>
 __global__ void __launch_bounds__(32 * kCombWarps)
     k_combine(const __grid_constant__ CombTable tab, const __grid_constant__ Scalars sc) {
+    using PT = Part<PREC>;
+    using T = typename PT::T;
     // Everything that does not come from the kernel before is read ahead of the
     // wait for it (this kernel is launched early and waits through most of the
     // previous one): the segment's place in the table and, in a step, the old
@@ -1014,18 +1044,18 @@ __global__ void __launch_bounds__(32 * kCombWarps)
     const double steps = step ? sc.state[TULA_STATE_STEPS] : 0.0;
     grid_dependency();
     if (!active) return;
-    const float2 *part = NA == kAcc ? sc.part1 : sc.part2;
-    float2 *spart = NA == kAcc ? sc.spart1 : sc.spart2;
+    const T *part = reinterpret_cast<const T *>(NA == kAcc ? sc.part1 : sc.part2);
+    T *spart = reinterpret_cast<T *>(NA == kAcc ? sc.spart1 : sc.spart2);
     unsigned *sctr = NA == kAcc ? sc.sctr1 : sc.sctr2;
 
     // The segment's tiles: lane i adds tiles i, i + 32, ... in order (8 loads in
     // flight), then a fixed tree across the warp.
-    float2 v[NA];
+    T v[NA];
 #pragma unroll
-    for (int a = 0; a < NA; ++a) v[a] = make_float2(0.f, 0.f);
+    for (int a = 0; a < NA; ++a) v[a] = PT::zero();
     int i = lane;
     for (; i + 7 * 32 < n; i += 8 * 32) {
-        float2 x[8][NA];
+        T x[8][NA];
 #pragma unroll
         for (int u = 0; u < 8; ++u)
 #pragma unroll
@@ -1033,11 +1063,11 @@ __global__ void __launch_bounds__(32 * kCombWarps)
 #pragma unroll
         for (int u = 0; u < 8; ++u)
 #pragma unroll
-            for (int a = 0; a < NA; ++a) v[a] = ff_add(v[a], x[u][a]);
+            for (int a = 0; a < NA; ++a) v[a] = PT::add(v[a], x[u][a]);
     }
     for (; i < n; i += 32) {
 #pragma unroll
-        for (int a = 0; a < NA; ++a) v[a] = ff_add(v[a], part[(first + i) * NA + a]);
+        for (int a = 0; a < NA; ++a) v[a] = PT::add(v[a], part[(first + i) * NA + a]);
     }
     warp_sums_ff<NA>(v);
 
@@ -1062,16 +1092,16 @@ __global__ void __launch_bounds__(32 * kCombWarps)
     }
     if (last_all) {
         fence_acq_rel();
-        finalize_step(sc, g2_prev, steps);
+        finalize_step<PREC>(sc, g2_prev, steps);
     }
     if (!last_seg) return;
     if (nseg > 1) {
         fence_acq_rel();
 #pragma unroll
-        for (int a = 0; a < NA; ++a) v[a] = make_float2(0.f, 0.f);
+        for (int a = 0; a < NA; ++a) v[a] = PT::zero();
         for (int j = lane; j < nseg; j += 32) {
 #pragma unroll
-            for (int a = 0; a < NA; ++a) v[a] = ff_add(v[a], __ldcg(&spart[(sg0 + j) * NA + a]));
+            for (int a = 0; a < NA; ++a) v[a] = PT::add(v[a], __ldcg(&spart[(sg0 + j) * NA + a]));
         }
         warp_sums_ff<NA>(v);
         if (lane == 0) sctr[tg] = 0u;  // re-arm
@@ -1079,11 +1109,10 @@ __global__ void __launch_bounds__(32 * kCombWarps)
 
     // This warp holds tensor tg's sums (lane 0).
     if constexpr (NA == kAcc) {
-        tensor_done(sc, tg, ff_to_double(v[0]), ff_to_double(v[1]), ff_to_double(v[2]),
-                    scale_old);
+        tensor_done(sc, tg, PT::value(v[0]), PT::value(v[1]), PT::value(v[2]), scale_old);
     } else {
         // lanes 0 and 1 take the two square roots in one instruction
-        const double sw = __shfl_sync(kFull, ff_to_double(v[0]), 0);
+        const double sw = __shfl_sync(kFull, PT::value(v[0]), 0);
         const double sg = sc.tsum[(size_t)tg * kTsum + 0];
         const double r = sqrt(lane == 0 ? sw : sg);
         const double nw = __shfl_sync(kFull, r, 0), ng = __shfl_sync(kFull, r, 1);
@@ -1512,7 +1541,7 @@ int launch_streaming(Kernel kernel, int n, const int64_t *numels, int chunk, int
 }
 
 // k_combine over all tensors (tiles of `chunk` elements), NA sums per tile.
-template <int NA>
+template <int NA, bool PREC>
 int launch_combine(int n, const int64_t *numels, int chunk, const Scalars &sc_in, cudaStream_t s) {
     std::unique_ptr<CombTable> tab(new CombTable);
     Scalars sc = sc_in;
@@ -1545,7 +1574,7 @@ int launch_combine(int n, const int64_t *numels, int chunk, const Scalars &sc_in
         tab->sfirst[cnt] = ns;
         s_global += ns;
         const int grid = (ns + kCombWarps - 1) / kCombWarps;
-        const int rc = launch_pdl(k_combine<NA>, grid, 32 * kCombWarps, 0, s, *tab, sc);
+        const int rc = launch_pdl(k_combine<NA, PREC>, grid, 32 * kCombWarps, 0, s, *tab, sc);
         if (rc) return rc;
     }
     return TULA_OK;
@@ -1605,7 +1634,7 @@ int run_reduce_k(int K, int n, const int64_t *numels, const Scalars &sc, int gri
                                           fill);
     if (rc) return rc;
     record(mid_event, s);
-    return launch_combine<kAcc>(n, numels, chunk, sc, s);
+    return launch_combine<kAcc, PR>(n, numels, chunk, sc, s);
 }
 
 template <bool WM, bool RW, bool SS, bool PR, typename Fill>
@@ -1791,7 +1820,7 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
 #undef TULA_UPD
     if (rc) return rc;
     record(hp->trace_events[3], s);
-    if (sw) rc = launch_combine<1>(n, numels, c2, sc, s);
+    if (sw) rc = launch_combine<1, false>(n, numels, c2, sc, s);
     if (rc) return rc;
     record(hp->trace_events[4], s);
     return TULA_OK;
