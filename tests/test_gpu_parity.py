@@ -26,10 +26,15 @@ def _built():
     T.lib()
 
 
-def _ragged_pset(extra=()):
+def _ragged_pset(extra=(), K=None):
+    """Empty, tiny and ragged tensors; with K, also sizes one below, at and one above a tile and
+    two tiles of either pass (the tile sizes the library uses for K replicas)."""
     ps = W.ParamSet("ragged")
-    for n in (0, 1, 3, 4, 5, 63, 64, 65, 4095, CHUNK - 1, CHUNK, CHUNK + 1, 40000, 100003,
-              *extra):
+    sizes = [0, 1, 3, 4, 5, 63, 64, 65, 4095, CHUNK - 1, CHUNK, CHUNK + 1, 40000, 100003, *extra]
+    if K is not None:
+        for t in (T.tula_ags_chunk_elems(1, K), T.tula_ags_chunk_elems(2, 3)):
+            sizes += [t - 1, t, t + 1, 2 * t + 1]
+    for n in sizes:
         ps.add((n,), W.KIND_NORMAL)
     return ps
 
@@ -52,7 +57,7 @@ def test_resnet20_ten_steps():
 def test_ragged_shapes(K, shift):
     """Tensors of 0..100003 elements (ragged chunk tails); shift=1 misaligns every tensor."""
     wl = W.workload("stress_k4", seed=11 + K, factor_range=(1e-3, 1e1), zero_patterns=False)
-    pair = Pair(wl, K=K, align=1 if shift else 64, shift=shift, pset=_ragged_pset())
+    pair = Pair(wl, K=K, align=1 if shift else 64, shift=shift, pset=_ragged_pset(K=K))
     # draw 1 twice (Delta = 0: scaled), then x2 (Delta = 3: unscaled), then a fresh draw
     for i, (seed_step, mult) in enumerate(((1, 1.0), (1, 1.0), (1, 2.0), (2, 1.0))):
         pair.step(seed_step, mult, refresh=(K > 1 and i == 0))
@@ -200,6 +205,39 @@ def _oracle_g2(buf, K):
         g = [buf.g[k][p].reshape(-1).cpu().numpy() for k in range(K)]
         total += O.sqnorm(O.replica_mean(g))
     return total
+
+
+def test_steps_replayed_from_a_cuda_graph():
+    """A captured step (no allocation, no host synchronisation, kernels chained by programmatic
+    dependent launch) replays to the same bytes as the same steps issued one by one."""
+    wl = W.workload("resnet18")
+    bufs, steps = [], []
+    for _ in range(2):
+        buf = W.allocate(wl, "cuda")
+        W.fill_state(buf, wl)
+        W.fill_grads(buf, wl, step=1)
+        bufs.append(buf)
+        steps.append(T.AGSOptimizerStep(buf.w, buf.g, buf.m, s_max=wl.smax))
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        for st in steps:  # one eager step each: the library sets itself up outside capture
+            st.step(wl.lr, wl.momentum, wl.weight_decay, refresh_scale=True, stream=s)
+    s.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        steps[1].step(wl.lr, wl.momentum, wl.weight_decay, stream=s)
+    for i in range(4):
+        with torch.cuda.stream(s):
+            steps[0].step(wl.lr, wl.momentum, wl.weight_decay, stream=s)
+            g.replay()
+        s.synchronize()
+        a, b = bufs
+        assert torch.equal(a.w_flat, b.w_flat) and torch.equal(a.m_flat, b.m_flat), i
+        assert torch.equal(a.g_flats[0], b.g_flats[0]), i
+        assert torch.equal(steps[0].state, steps[1].state), i
+        assert torch.equal(steps[0].stats, steps[1].stats), i
+    assert steps[0].state[1].item() == 5.0  # five steps taken: the refresh step and four more
 
 
 @pytest.mark.parametrize("name", ["stress_k1", "stress_k4", "stress_k16"])
