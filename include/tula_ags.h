@@ -29,10 +29,15 @@
  *     library leaves it re-usable (its counters back at zero) after every
  *     call.  Calls that share a workspace must be ordered (one stream).
  *   - Return value: TULA_OK (0) or a negative TULA_ERR_* code.  Argument
- *     errors are detected on the host before anything is enqueued.
+ *     errors are detected on the host before anything is enqueued.  After
+ *     TULA_ERR_CUDA (a launch failed part way) or a nonzero
+ *     tula_ags_workspace_error() (a bounded wait inside a kernel ran out), the
+ *     step may be partly applied: zero the workspace again before reusing it.
  *   - Element-wise arithmetic is IEEE fp32, one rounding per operation, in the
- *     order written below (no fused multiply-add).  Norms are fp64 sums of
- *     fp32 partial sums of squares.
+ *     order written below (no fused multiply-add).  Squared norms are fp32 sums
+ *     within a tile (<= 2688 elements) added across tiles as float-float pairs
+ *     (~48 significant bits); norms that feed a coefficient (gradscale refresh,
+ *     LARS) add exact fp64 squares in fp64 throughout.
  */
 #ifndef TULA_AGS_H
 #define TULA_AGS_H
