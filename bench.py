@@ -88,6 +88,12 @@ def pass2_bytes_per_param(with_momentum=True) -> int:
     return 20 if with_momentum else 12
 
 
+def step_design_bytes_per_param(K: int) -> int:
+    """What the two passes move as built: pass 1 plus pass 2 (the mean is written over
+    replica 0 and read back by the update, as an in-place all-reduce would leave it)."""
+    return pass1_bytes_per_param(K) + pass2_bytes_per_param()
+
+
 def step_min_bytes_per_param(K: int) -> int:
     """Algorithmic minimum of one step: read K replicas, w, m; write w, m."""
     return 4 * K + 16
@@ -436,7 +442,9 @@ def run_ours(args, wl):
                        "after_update": statistics.fmean(t_cmb2)},
         "step_hbm": {"algorithmic_bytes_per_param": step_min_bytes_per_param(K),
                      "achieved_gbs": step_gbs, "frac": step_gbs / peak,
-                     "frac_of_8tbs": step_gbs / 8000.0},
+                     "frac_of_8tbs": step_gbs / 8000.0,
+                     "design_bytes_per_param": step_design_bytes_per_param(K),
+                     "design_gbs": step_design_bytes_per_param(K) * N / (ms_per_step / 1e3) / 1e9},
         "e2e": e2e,
         "gpu_launches": launches,
         "clocks": clocks,
