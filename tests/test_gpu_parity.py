@@ -143,6 +143,7 @@ def test_bitwise_reproducible_across_runs_and_grids(name):
         st = T.AGSOptimizerStep(buf.w, buf.g, buf.m, grid_ctas=grid)
         st.state.copy_(torch.tensor([1.0, 3.0, 0.0, 0.0], dtype=torch.float64))
         st.step(wl.lr, wl.momentum, wl.weight_decay, refresh_scale=True)
+        st.step(wl.lr, wl.momentum, wl.weight_decay)  # and a step without refresh
         torch.cuda.synchronize()
         outs.append([buf.g_flats[0].clone(), buf.w_flat.clone(), buf.m_flat.clone(),
                      st.stats.clone(), st.state.clone(), st.scale.clone()])
