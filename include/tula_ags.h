@@ -198,8 +198,8 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
  * that array until the process exits.  hp->workspace and hp->workspace_bytes are ignored.
  *
  * Limit: the scratch a tensor list needs (tula_ags_workspace_size) is about 110 bytes per tensor
- * plus, per 1000 parameters, 13 bytes (K <= 2), 20 (K = 4), 31 (K = 8) or 67 (K = 16): e.g. 4096
- * tensors holding up to ~1.3e9 parameters at K <= 2, ~5.4e8 at K = 8, ~2.5e8 at K = 16.  A larger
+ * plus, per 1000 parameters, 14 bytes (K <= 2), 21 (K = 4), 32 (K = 8) or 68 (K = 16): e.g. 4096
+ * tensors holding up to ~1.2e9 parameters at K <= 2, ~5.1e8 at K = 8, ~2.4e8 at K = 16.  A larger
  * list is rejected with TULA_ERR_SCRATCH_LIMIT before anything is enqueued.
  *
  * Set-up: the first call on each device, with that device current, looks up the array's device
