@@ -1,31 +1,32 @@
 // libtula_ags: the AGS optimizer step (Tula, arXiv 2603.18112) for sm_103a.
 //
-// Per step, three kernels on the caller's stream, chained by programmatic
+// Per step, four kernels on the caller's stream, chained by programmatic
 // dependent launch so that each one's launch and prologue overlap the tail of
 // the one before:
 //
 //   k_reduce   (pass 1)  K-way replica mean (Eq. 1c) written over replica 0, and
-//                        fp64 per-tile partial sums of |gbar|^2, |g_0|^2 [, |w|^2].
+//                        per-tile partial sums of |gbar|^2, |g_0|^2 [, |w|^2].
 //   k_combine            per tensor, the fixed-order sum of its tile partials,
 //                        its statistics, its coefficient when scaled (the old
 //                        gradscale, Eq. 8's s, or the LARS ratio) and, when
 //                        asked, the refreshed gradscale (UpdateGradScale,
-//                        Algorithm 1); the CTA finishing last forms |G|^2,
-//                        Delta (Eq. 5) and the branch of Algorithm 1.
+//                        Algorithm 1); the warp taking the last segment ticket
+//                        forms |G|^2, Delta (Eq. 5) and the branch of Algorithm 1.
 //   k_update   (pass 2)  d = c gbar + wd w; m = mu m + d; w = w - lr m (Eq. 7b with
-//                        the wrapped SGD); |w|^2 per tile for the statistics
-//                        (then a k_combine of those).
+//                        the wrapped SGD); |w|^2 per tile for the statistics,
+//   k_combine            then summed per tensor.
 //
 // The streaming passes: each tensor is cut into tiles of T elements (T fixed
 // per pass by how many tensors it streams, so that one tile of every stream
-// fills a 32 KB shared-memory stage).  One persistent CTA per SM takes tiles
-// round-robin.  Its producer warp moves tiles from HBM into a 6-stage ring
-// with TMA bulk copies (cp.async.bulk ... mbarrier::complete_tx), one copy per
-// stream issued by one lane each, so up to 192 KB per SM are in flight; three
-// consumer warps, each owning two stages, compute from shared memory and
-// release the stage through an mbarrier.  Consumers keep fp64 partial sums
-// per lane and reduce four tiles' worth at a time across the warp in a fixed
-// tree, so the FP64 latency chains overlap.  Only plain stores leave a tile.
+// fills one shared-memory stage: 32 KB in pass 1, 24 KB in pass 2).  One
+// persistent CTA per SM; small launches deal tiles round-robin, larger ones
+// claim them from a global counter (SMs stream at unequal rates).  The producer
+// warp moves tiles from HBM into the stage ring with TMA bulk copies
+// (cp.async.bulk ... mbarrier::complete_tx), one copy per stream issued by one
+// lane each; consumer warps, each owning whole stages, compute from shared
+// memory and release the stage through an mbarrier.  Tile partials are fp32
+// sums within a tile, carried as float-float pairs (fp64 in the precise mode
+// for norms that feed a coefficient); only plain stores leave a tile.
 //
 // Every mbarrier wait is bounded; a wait that runs out sets an error word in
 // the workspace (tula_ags_workspace_error) and the CTA drains its copies in
@@ -33,8 +34,9 @@
 // 20-70 bytes); nothing here is a contraction, so no tensor cores.  The tile
 // table, pointers and sizes travel in the kernel parameter block
 // (__grid_constant__, up to ~31 KB per launch): no host-to-device copy,
-// allocation or host sync is ever needed.  The reduction order depends on the
-// numels only, so results are bitwise reproducible and independent of the grid.
+// allocation or host sync is ever needed.  Each tile's partials go to the
+// tile's own slot and are summed in an order fixed by the numels, so results
+// are bitwise reproducible and independent of the grid.
 #include "tula_ags.h"
 
 #include <cuda_runtime.h>

@@ -16,7 +16,7 @@ from paper_2603_18112_gb300 import workloads as W
 
 pytestmark = pytest.mark.gpu
 
-CHUNK = 16384
+CHUNK = 16384  # an arbitrary ragged boundary; the tile sizes themselves come from the library
 
 
 @pytest.fixture(scope="module", autouse=True)
