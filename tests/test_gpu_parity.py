@@ -241,6 +241,45 @@ def test_steps_replayed_from_a_cuda_graph():
     assert steps[0].state[1].item() == 5.0  # five steps taken: the refresh step and four more
 
 
+def test_largest_tensor_the_library_takes():
+    """One tensor at the per-tensor limit (K = 2: 1,694,208 tiles of 1536 elements, 2.6e9
+    elements, past 2^31), constant per role so that every element has the same closed-form
+    result, which the oracle gives on a few elements: sampled elements around 2^31 and at both
+    ends, the extremes over the whole tensor, and |G|^2 = n |gbar|^2."""
+    K = 2
+    n = 1_694_208 * min(T.tula_ags_chunk_elems(1, K + 1), T.tula_ags_chunk_elems(2, 4))
+    assert n > 2 ** 31
+    need = (K + 2) * 4 * n + (1 << 30)
+    if torch.cuda.mem_get_info()[0] < need:
+        pytest.skip(f"needs {need / 1e9:.0f} GB of device memory")
+    vals = {"w": 0.5, "m": 0.01, "g0": 0.003, "g1": -0.001}
+    w = torch.full((n,), vals["w"], device="cuda")
+    m = torch.full((n,), vals["m"], device="cuda")
+    g = [torch.full((n,), vals["g0"], device="cuda"), torch.full((n,), vals["g1"], device="cuda")]
+    st = T.AGSOptimizerStep([w], [[g[0]], [g[1]]], [m])
+    lr, mu, wd = 0.1, 0.9, 5e-4
+    st.step(lr, mu, wd)
+    torch.cuda.synchronize()
+
+    # the oracle on four elements of the same values
+    w_h = [np.full(4, vals["w"], np.float32)]
+    m_h = [np.full(4, vals["m"], np.float32)]
+    g_h = [[np.full(4, vals["g0"], np.float32)], [np.full(4, vals["g1"], np.float32)]]
+    state_h = O.new_state()
+    O.ags_step(w_h, m_h, g_h, lr, mu, wd, O.OracleHP(K=K), scale=np.ones(1, np.float32),
+               state=state_h)
+    idx = torch.tensor([0, 1, 2 ** 31 - 1, 2 ** 31, 2 ** 31 + 1, n // 2, n - 2, n - 1],
+                       device="cuda")
+    for got, want, what in ((w, w_h[0][0], "w"), (m, m_h[0][0], "m"), (g[0], g_h[0][0][0], "mean")):
+        assert torch.all(got[idx] == float(want)), what
+        assert got.min().item() == float(want) and got.max().item() == float(want), what
+    gbar = float(g_h[0][0][0])
+    g2 = st.state[0].item()
+    assert g2 == pytest.approx(n * gbar * gbar, rel=1e-5)
+    assert st.stats[0, T.TULA_STAT_G_SQ].item() == pytest.approx(n * gbar * gbar, rel=1e-5)
+    assert st.state[3].item() == 0.0  # the first step is unscaled
+
+
 @pytest.mark.parametrize("name", ["stress_k1", "stress_k4", "stress_k16"])
 def test_stress_full_size_sampled(name):
     """The ~1.65e9-element stress set at full size, in the benchmark's launch shape: |G|^2
