@@ -243,6 +243,16 @@ int tula_ags_plan_chunks(const int64_t *numels, int n_tensors, int chunk_elems,
                          int64_t *chunk_start_out);
 
 /*
+ * Failure-detection check: launches, on `stream`, one warp that makes the library's bounded
+ * mbarrier wait run out (it waits on an mbarrier that nothing arrives on; about two seconds) and
+ * records it in the workspace's error word exactly as a streaming kernel records a stage that
+ * never fills.  tula_ags_workspace_error() then reports bit 0; the CUDA context stays usable.
+ * No counterpart in the paper.  TULA_ERR_WORKSPACE when workspace is NULL, misaligned or smaller
+ * than the error word's offset + 4 bytes.
+ */
+int tula_ags_check_wait_timeout(void *workspace, size_t workspace_bytes, void *stream);
+
+/*
  * Reads (synchronously, with cudaMemcpy) and clears the workspace's error word: 0 when every
  * wait of the kernels that used this workspace completed; bit 0 set when a bounded wait inside a
  * kernel ran out (the step's results are then not valid).  numels, n_tensors and K are those the

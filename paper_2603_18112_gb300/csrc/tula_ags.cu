@@ -87,7 +87,7 @@ constexpr int kParamBudget = 31 * 1024; // kernel parameter bytes per launch (li
 constexpr int kAcc = 3;                 // partial sums per pass-1 tile: |gbar|^2, |g_0|^2, |w|^2
 constexpr int kTsum = 4;                // per-tensor sums (stride)
 constexpr unsigned kFull = 0xffffffffu;
-constexpr uint32_t kSpinLimit = 1u << 22;  // bound on every mbarrier wait (>= 1 s)
+constexpr uint32_t kSpinLimit = 1u << 19;  // bound on every mbarrier wait (~2 s on GB300)
 
 enum Mode { kModeStep = 0, kModeStats = 1, kModeScale = 2, kModeUpdate = 3 };
 
@@ -1322,6 +1322,20 @@ __device__ __forceinline__ float scale1(float gs, float gl, const Scalars &sc) {
     return fminf(fabsf(__fdiv_rn(gs, __fadd_rn(gl, sc.eps))), sc.s_max);
 }
 
+// The bounded wait itself, on an mbarrier that nothing ever arrives on: the
+// wait runs out and the kernel reports it in the error word, the way every
+// streaming kernel reports a stage that never fills.  (Failure detection is
+// checked with this, not with a real fault.)
+__global__ void __launch_bounds__(32) k_wait_check(unsigned *err) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        mbar_fence_init();
+    }
+    __syncwarp();
+    if (threadIdx.x == 0 && !mbar_wait(&bar, 0u)) atomicOr(err, 1u);
+}
+
 constexpr int kScaleThreads = 128;
 
 __global__ void __launch_bounds__(kScaleThreads)
@@ -1708,6 +1722,21 @@ int tula_ags_plan_chunks(const int64_t *numels, int n_tensors, int chunk_elems,
         c += tiles_of(numels[p], chunk_elems);
     }
     chunk_start_out[n_tensors] = c;
+    return TULA_OK;
+}
+
+int tula_ags_check_wait_timeout(void *workspace, size_t workspace_bytes, void *stream) {
+    const WsLayout L = ws_layout(1, Plan{});
+    if (!workspace || workspace_bytes < L.err + sizeof(unsigned)) return TULA_ERR_WORKSPACE;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return TULA_ERR_WORKSPACE;
+    unsigned *err = reinterpret_cast<unsigned *>(static_cast<char *>(workspace) + L.err);
+    k_wait_check<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(err);
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) {
+        g_last_cuda = (int)e;
+        return TULA_ERR_CUDA;
+    }
     return TULA_OK;
 }
 

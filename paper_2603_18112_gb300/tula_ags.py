@@ -89,9 +89,10 @@ def lib() -> ctypes.CDLL:
     L.tula_ags_chunk_elems.restype = c_int
     L.tula_ags_workspace_error.argtypes = [c_void_p, c_size_t, i64p, c_int, c_int,
                                            ctypes.POINTER(c_int)]
+    L.tula_ags_check_wait_timeout.argtypes = [c_void_p, c_size_t, c_void_p]
     for name in ("tula_ags_workspace_size", "tula_ags_step", "tula_layer_stats",
                  "tula_ags_update_scale", "tula_ags_plan_chunks", "tula_ags_step_static_scratch",
-                 "tula_ags_workspace_error"):
+                 "tula_ags_workspace_error", "tula_ags_check_wait_timeout"):
         getattr(L, name).restype = c_int
     _lib = L
     return L
@@ -161,6 +162,15 @@ def tula_ags_launch_count() -> int:
 def tula_ags_chunk_elems(pass_: int, streams: int) -> int:
     """Elements per tile of pass 1 (reduction) or pass 2 (update) with `streams` streams."""
     return lib().tula_ags_chunk_elems(pass_, streams)
+
+
+def tula_ags_check_wait_timeout(workspace: torch.Tensor, stream=None) -> None:
+    """Launches the bounded-wait check (about a second on the GPU): afterwards the workspace's
+    error word has bit 0 set, as after a stage that never filled."""
+    _check(lib().tula_ags_check_wait_timeout(c_void_p(workspace.data_ptr()),
+                                             workspace.numel() * workspace.element_size(),
+                                             _stream_ptr(stream)),
+           "tula_ags_check_wait_timeout")
 
 
 def tula_ags_workspace_error(workspace: torch.Tensor, numels, K: int) -> int:

@@ -342,3 +342,24 @@ def test_stress_full_size_sampled(name):
         assert_norm_close(gpu.scale.cpu().numpy()[sample], scale_h, name + " scale")
     del buf, gpu
     torch.cuda.empty_cache()
+
+
+def test_a_wait_that_runs_out_is_reported_and_the_context_survives():
+    """Failure detection without a fault: the library's bounded mbarrier wait, on a barrier
+    nothing arrives on, gives up (about a second), sets the workspace's error word, and the
+    next step on the same context runs and matches the oracle."""
+    import time
+    wl = W.workload("resnet20")
+    pair = Pair(wl)
+    numels = [t.numel() for t in pair.buf.w]
+    ws = pair.gpu.workspace
+    assert T.tula_ags_workspace_error(ws, numels, pair.K) == 0
+    t0 = time.perf_counter()
+    T.tula_ags_check_wait_timeout(ws)
+    torch.cuda.synchronize()
+    waited = time.perf_counter() - t0
+    assert T.tula_ags_workspace_error(ws, numels, pair.K) == 1  # reported, then cleared
+    assert T.tula_ags_workspace_error(ws, numels, pair.K) == 0
+    assert 0.05 < waited < 60.0
+    pair.step(1, 1.0)  # the context is still usable and the step still exact
+    assert T.tula_ags_workspace_error(ws, numels, pair.K) == 0
