@@ -512,8 +512,9 @@ struct TensorCache {
 // stage's full barrier is armed (the barrier's release/acquire orders it), and
 // -1 there tells a consumer that no tile is left.  Lane i < ns of the producer
 // fetches stream i's pointer (role roles[i]) and issues that stream's copy to
-// offset i * chunk floats of the stage.  With `reverse` the order is mirrored
-// (pass 2 walks the tiles backwards, so it starts on what pass 1 left in L2).
+// offset i * chunk floats of the stage.  Both passes walk the tiles in the same
+// order (measured: walking pass 2 backwards, to start on the mean pass 1 wrote
+// last, was 1 % slower per step).
 
 __device__ __forceinline__ unsigned claim_tiles(unsigned *ctr, unsigned n) {
     return atomicAdd(ctr, n);
@@ -526,15 +527,12 @@ __device__ __forceinline__ int static_tiles(int nc) {
     return b < nc ? (nc - b + g - 1) / g : 0;
 }
 __device__ __forceinline__ bool claims_tiles(int nc) { return nc >= kDynTiles * (int)gridDim.x; }
-__device__ __forceinline__ int static_tile(int nc, int j, bool reverse) {
-    const int i = (int)blockIdx.x + j * (int)gridDim.x;
-    return reverse ? nc - 1 - i : i;
-}
+__device__ __forceinline__ int static_tile(int j) { return (int)blockIdx.x + j * (int)gridDim.x; }
 
 template <typename R, int NP, int NS>
 __device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
                                         const int (&roles)[NS], int ns, int chunk,
-                                        int js, unsigned *ctr, bool reverse, uint32_t ring,
+                                        int js, unsigned *ctr, uint32_t ring,
                                         uint64_t *full, uint64_t *empty, int *stage_tile) {
     const int lane = threadIdx.x & 31;
     const int role = lane < ns ? roles[lane] : 0;
@@ -595,7 +593,7 @@ __device__ __forceinline__ void produce(const Table<NP> &tab, const Scalars &sc,
             issued = j + 1;
             continue;
         }
-        const int c = reverse ? (int)(nc - 1u - i) : (int)i;
+        const int c = (int)i;
         const TilePos q = tc.at(tab, c, chunk, role, ns);
         const uint32_t bytes = 16u * (uint32_t)tc.nv;
         if (lane == 0) {
@@ -838,8 +836,8 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
     if (RW) roles[ns++] = KS;
     if (SS) roles[ns++] = KS + 1;
     if (warp == 0) {
-        produce<Ring1, P1<KT>::NP, NSMAX>(tab, sc, roles, ns, chunk, js, sc.tiles, false, ring, full,
-                                   empty, stage_tile);
+        produce<Ring1, P1<KT>::NP, NSMAX>(tab, sc, roles, ns, chunk, js, sc.tiles, ring, full,
+                                          empty, stage_tile);
         return;
     }
     if (early) grid_wait();
@@ -863,7 +861,7 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
             }
             if (stop) continue;
             // A round-robin tile is located before its wait, a claimed one after.
-            int c = j < js ? static_tile(tab.nc, j, false) : -1;
+            int c = j < js ? static_tile(j) : -1;
             TilePos q;
             if (c >= 0) q = tc.at(tab, c, chunk, my_role, ns);
             const int got = next_tile<Ring1>(sc, j, full, stage_tile);
@@ -1132,7 +1130,6 @@ __global__ void __launch_bounds__(32 * kCombWarps)
 // ----------------------------------------------------------------------------
 // Pointer roles: 0 = gbar, 1 = w, 2 = m, 3 = per-element gradscale.
 // Stage streams: gbar, w, then m (HM), then the per-element scale (PE, scaled).
-// Tiles run in reverse order: the mean pass 1 wrote last is still in L2.
 
 constexpr int kNP2 = 4;
 
@@ -1189,8 +1186,8 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
     if (!HM) roles[2] = 3;
     if (warp == 0) {
         const bool se = PE && sc.flags[0];
-        produce<Ring2, kNP2, 4>(tab, sc, roles, 2 + (HM ? 1 : 0) + (se ? 1 : 0), chunk, js, sc.tiles + 2,
-                         true, ring, full, empty, stage_tile);
+        produce<Ring2, kNP2, 4>(tab, sc, roles, 2 + (HM ? 1 : 0) + (se ? 1 : 0), chunk, js,
+                                sc.tiles + 2, ring, full, empty, stage_tile);
         return;
     }
     if (early) grid_wait();
@@ -1219,7 +1216,7 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
             ptile[p] = -1;
             pend[p] = 0.f;
             if (stop) continue;
-            int c = j < js ? static_tile(tab.nc, j, true) : -1;
+            int c = j < js ? static_tile(j) : -1;
             TilePos q;
             if (c >= 0) q = tc.at(tab, c, chunk, my_role, ns);
             const int got = next_tile<Ring2>(sc, j, full, stage_tile);
@@ -1509,12 +1506,12 @@ int launch_pdl(void (*kernel)(KArgs...), int grid, int threads, int smem, cudaSt
 }
 
 // Splits tensors [0, n) into parameter blocks of tiles of `chunk` elements and
-// launches `kernel` once per block (in reverse block order when `reverse`).
+// launches `kernel` once per block.
 // fill(p, ptrs) writes tensor p's pointers.
 template <int NP, typename Kernel, typename Fill>
 int launch_streaming(Kernel kernel, int n, const int64_t *numels, int chunk, int threads,
                      int smem, const Scalars &sc, int grid_override, cudaStream_t stream,
-                     Fill fill, bool reverse = false) {
+                     Fill fill) {
     using T = Table<NP>;
     const int grid_cap = resident_ctas((const void *)kernel, threads, smem);
     if (grid_cap <= 0) {
@@ -1545,7 +1542,6 @@ int launch_streaming(Kernel kernel, int n, const int64_t *numels, int chunk, int
         c_global += nc;
         tabs.push_back(std::move(tab));
     }
-    if (reverse) std::reverse(tabs.begin(), tabs.end());
     tabs.front()->first = 1;
     for (const auto &tab : tabs) {
         int grid = grid_override > 0 ? grid_override : grid_cap;
@@ -1798,9 +1794,10 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
     Scalars sc = make_scalars(hp, K, n, hp->workspace, L, kModeStep);
     const bool lars = hp->rule == TULA_RULE_LARS;
     sc.read_w = lars ? 1 : 0;
-    // When the mean fits in L2, the replica loads of pass 1 are marked to leave
-    // L2 first, so that pass 2 (which walks the tiles backwards) finds much of
-    // the mean still there.  For larger models the mark only costs bandwidth.
+    // When the mean fits in L2, every bulk load is marked to leave L2 first, so
+    // that the lines the step writes (the mean, w, m), which the update and the
+    // next step read again, stay there instead (ResNet-18 K = 4: 103 -> 79 us per
+    // step).  For larger models the mark only costs bandwidth.
     long long n_total = 0;
     for (int p = 0; p < n; ++p) n_total += numels[p];
     sc.evict_first = (K > 1 && 4 * n_total <= l2_bytes()) ? 1 : 0;
@@ -1840,7 +1837,7 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
     sc.mode = kModeUpdate;
 #define TULA_UPD(HM, PE, SW)                                                                \
     launch_streaming<kNP2>(k_update<HM, PE, SW>, n, numels, c2, Ring2::kThreads,             \
-                           Ring2::kSmemBytes, sc, hp->grid_ctas, s, fill2, true)
+                           Ring2::kSmemBytes, sc, hp->grid_ctas, s, fill2)
     if (hm) {
         if (per_elem) rc = sw ? TULA_UPD(true, true, true) : TULA_UPD(true, true, false);
         else rc = sw ? TULA_UPD(true, false, true) : TULA_UPD(true, false, false);
