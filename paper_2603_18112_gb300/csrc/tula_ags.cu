@@ -322,10 +322,6 @@ __device__ __forceinline__ void grid_wait() { asm volatile("griddepcontrol.wait;
 __device__ __forceinline__ void grid_launch_dependents() {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
-__device__ __forceinline__ void grid_dependency() {
-    grid_wait();
-    grid_launch_dependents();
-}
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p) {
     return (uint32_t)__cvta_generic_to_shared(p);
@@ -813,11 +809,15 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
     constexpr int KS = P1<KT>::KS;
     constexpr int NSMAX = KS + 2;
     extern __shared__ __align__(128) unsigned char smem[];
-    // In a step that does not read w, the kernels still running before this one
-    // (the previous step's update and combine) write nothing this kernel loads:
-    // the producer of the pass's first launch streams replicas in right away,
-    // and only the consumers, which write the mean over replica 0 and the tile
-    // partials, wait for them.  Otherwise the whole CTA waits first.
+    // In a step that does not read w, the first launch of the pass starts at
+    // once.  It can only have been started early by the previous step's pass-2
+    // combine (the update triggers its successor only when that combine
+    // follows), and that combine starts it after its own wait, i.e. once the
+    // previous update has completed: nothing still running then reads the
+    // replicas or the pass-1 partials this kernel writes, and nothing writes
+    // what it loads.  The running combine reads the per-tensor sums the next
+    // combine writes, so this kernel does not complete before it (one wait per
+    // CTA at the end).  Otherwise the whole CTA waits first.
     grid_launch_dependents();
     const bool early = !RW && !SS && sc.mode == kModeStep && tab.first;
     if (!early) grid_wait();
@@ -840,7 +840,6 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
                                           empty, stage_tile);
         return;
     }
-    if (early) grid_wait();
     const int my_role = lane < ns ? roles[lane] : 0;
 
     const int cw = warp - 1;
@@ -905,6 +904,7 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
         }
         if (stop) break;
     }
+    if (early && threadIdx.x == 32) grid_wait();  // see the top of the kernel
 }
 
 // ----------------------------------------------------------------------------
@@ -1042,7 +1042,12 @@ __global__ void __launch_bounds__(32 * kCombWarps)
     const float scale_old = (active && step && sc.scale) ? sc.scale[tg] : 1.0f;
     const double g2_prev = step ? sc.state[TULA_STATE_G2_PREV] : 0.0;
     const double steps = step ? sc.state[TULA_STATE_STEPS] : 0.0;
-    grid_dependency();
+    grid_wait();
+    // Inside a step the successor (the update, or the next step's reduction)
+    // may start now; after tula_layer_stats or tula_ags_update_scale it starts
+    // when this kernel has completed (a step's reduction that starts early
+    // overwrites the tile partials this kernel reads).
+    if (sc.mode == kModeStep || NA == 1) grid_launch_dependents();
     if (!active) return;
     const T *part = reinterpret_cast<const T *>(NA == kAcc ? sc.part1 : sc.part2);
     T *spart = reinterpret_cast<T *>(NA == kAcc ? sc.spart1 : sc.spart2);
@@ -1171,7 +1176,10 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
     // whole CTA waits per element (the producer's stream count depends on the
     // branch) and in later launches of the pass (which share the tile counter
     // with the launch before).
-    grid_launch_dependents();
+    // Successors may start early only when the pass-2 combine follows (it waits
+    // for this kernel); the next step's reduction, when it follows directly,
+    // must start after this kernel has completed (see k_reduce).
+    if (SW) grid_launch_dependents();
     const bool early = !PE && tab.first;
     if (!early) grid_wait();
     uint64_t *full, *empty;
@@ -1337,7 +1345,7 @@ constexpr int kScaleThreads = 128;
 
 __global__ void __launch_bounds__(kScaleThreads)
     k_scale_elem(const __grid_constant__ Table<kNP3> tab, const __grid_constant__ Scalars sc) {
-    grid_dependency();
+    grid_wait();  // no early start for the successor: it may overwrite what this kernel reads
     const int lane = threadIdx.x & 31;
     const int warp = (int)((blockIdx.x * (unsigned)kScaleThreads + threadIdx.x) >> 5);
     const int nwarps = (int)((gridDim.x * (unsigned)kScaleThreads) >> 5);
