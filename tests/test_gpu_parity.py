@@ -363,3 +363,51 @@ def test_a_wait_that_runs_out_is_reported_and_the_context_survives():
     assert 0.05 < waited < 60.0
     pair.step(1, 1.0)  # the context is still usable and the step still exact
     assert T.tula_ags_workspace_error(ws, numels, pair.K) == 0
+
+
+@pytest.mark.parametrize("K", [1, 4])
+def test_calls_back_to_back_on_one_workspace_and_stream(K):
+    """A step, tula_layer_stats, a step, tula_ags_update_scale and a step issued on one stream
+    and one workspace with no synchronisation between them (a step's first kernels start before
+    the call ahead of them has completed) give what the oracle gives for the same sequence."""
+    wl = W.workload("stress_k4", seed=71 + K, factor_range=(1e-2, 1e1), zero_patterns=False)
+    pair = Pair(wl, K=K, pset=_ragged_pset(K=K))
+    buf, gpu = pair.buf, pair.gpu
+    W.fill_grads(buf, wl, step=1)
+    g_h = [W.to_numpy(buf.g[k]) for k in range(K)]
+    small = torch.empty_like(buf.g_flats[0])
+    W.fill_small(buf, wl, small, step=1)
+    small_views = W._views(small, buf.offsets, buf.pset.shapes, buf.numels)
+    small_h = W.to_numpy(small_views)
+    stats_mid = torch.zeros(pair.n, T.TULA_STATS_LEN, dtype=torch.float64, device="cuda")
+    hp = T.tula_ags_default_hparams(1)
+    hp.s_max = pair.s_max
+    hp.scale = gpu.scale.data_ptr()
+    hp.workspace, hp.workspace_bytes = gpu.workspace.data_ptr(), gpu.workspace.numel()
+    lr, mu, wd = wl.lr, pair.momentum, wl.weight_decay
+    torch.cuda.synchronize()
+    gpu.step(lr, mu, wd)
+    T.tula_layer_stats(buf.w, buf.g, stats_mid, gpu.workspace)
+    gpu.step(lr, mu, wd)
+    T.tula_ags_update_scale(small_views, buf.g[0], hp)
+    gpu.step(lr, mu, wd)
+    torch.cuda.synchronize()
+
+    def oracle_step():
+        return O.ags_step(pair.w_h, pair.m_h, g_h, lr, mu, wd, pair.hp, scale=pair.scale_h,
+                          state=pair.state_h)
+
+    oracle_step()
+    stats_mid_h = O.layer_stats(pair.w_h, g_h)
+    oracle_step()
+    O.update_scale(small_h, g_h[0], pair.hp.eps, pair.s_max, O.GRAN_TENSOR, scale=pair.scale_h)
+    stats_h = oracle_step()
+
+    assert_stats_close(stats_mid.cpu().numpy(), stats_mid_h, "layer_stats between steps")
+    assert_norm_close(gpu.scale.cpu().numpy(), pair.scale_h, "scale refreshed between steps")
+    assert_state_close(gpu.state.cpu().numpy(), pair.state_h, "state after three steps")
+    assert_stats_close(gpu.stats.cpu().numpy(), stats_h, "stats of the third step")
+    for p in range(pair.n):
+        assert np.array_equal(buf.g[0][p].reshape(-1).cpu().numpy(), g_h[0][p]), p
+        assert_f32_close(buf.w[p].reshape(-1).cpu().numpy(), pair.w_h[p], f"w[{p}]")
+        assert_f32_close(buf.m[p].reshape(-1).cpu().numpy(), pair.m_h[p], f"m[{p}]")
