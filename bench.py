@@ -47,6 +47,11 @@ def _args():
                     help="untimed load before the timed steps, so clock samples see load")
     ap.add_argument("--cpu-sample-s", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--step-kind", default="ags", choices=list(STEP_KINDS),
+                    help="ags: Algorithm 1 steps (the gradscale refreshed once, in warm-up); "
+                         "refresh: every step also refreshes the gradscale (UpdateGradScale fused "
+                         "into pass 1, precise norms); lars: the LARS rule (precise norms, w read "
+                         "in pass 1)")
     return ap.parse_args()
 
 
@@ -78,9 +83,14 @@ def job_throughput(params_per_rank: int, steps: int, world_size: int, t_max_ms: 
 # bytes per parameter (fp32)
 # ---------------------------------------------------------------------------
 
-def pass1_bytes_per_param(K: int) -> int:
-    """Reduction pass: read K replicas, write the mean over replica 0 (K > 1)."""
-    return 4 * K + (4 if K > 1 else 0)
+LARS_TRUST = 1e-3  # trust coefficient of the LARS steps timed here
+# step kind -> (reads w in pass 1, refreshes the gradscale every step)
+STEP_KINDS = {"ags": (False, False), "refresh": (False, True), "lars": (True, False)}
+
+
+def pass1_bytes_per_param(K: int, read_w: bool = False) -> int:
+    """Reduction pass: read K replicas (and w for LARS), write the mean over replica 0 (K > 1)."""
+    return 4 * K + (4 if K > 1 else 0) + (4 if read_w else 0)
 
 
 def pass2_bytes_per_param(with_momentum=True) -> int:
@@ -88,15 +98,16 @@ def pass2_bytes_per_param(with_momentum=True) -> int:
     return 20 if with_momentum else 12
 
 
-def step_design_bytes_per_param(K: int) -> int:
+def step_design_bytes_per_param(K: int, read_w: bool = False) -> int:
     """What the two passes move as built: pass 1 plus pass 2 (the mean is written over
     replica 0 and read back by the update, as an in-place all-reduce would leave it)."""
-    return pass1_bytes_per_param(K) + pass2_bytes_per_param()
+    return pass1_bytes_per_param(K, read_w) + pass2_bytes_per_param()
 
 
-def step_min_bytes_per_param(K: int) -> int:
-    """Algorithmic minimum of one step: read K replicas, w, m; write w, m."""
-    return 4 * K + 16
+def step_min_bytes_per_param(K: int, read_w: bool = False) -> int:
+    """Algorithmic minimum of one step: read K replicas, w, m; write w, m (LARS: w is read
+    once more, since its norm sets the coefficient before the update)."""
+    return 4 * K + 16 + (4 if read_w else 0)
 
 
 # ---------------------------------------------------------------------------
@@ -225,11 +236,13 @@ def _host_inputs(wl, frac=1.0):
     return pset, w, m, g
 
 
-def _oracle_steps(wl, w, m, g, steps):
+def _oracle_steps(wl, w, m, g, steps, kind="ags"):
     import numpy as np
 
     import oracle as O
-    hp = O.OracleHP(K=wl.K, s_max=wl.smax)
+    hp = O.OracleHP(K=wl.K, s_max=wl.smax, rule=O.RULE_LARS if kind == "lars" else O.RULE_AGS,
+                    lars_trust=LARS_TRUST)
+    hp.refresh_scale = kind == "refresh"
     scale = np.ones(len(w), np.float32)
     state = O.new_state()
     t0 = time.perf_counter()
@@ -238,13 +251,13 @@ def _oracle_steps(wl, w, m, g, steps):
     return time.perf_counter() - t0
 
 
-def cpu_baseline(wl, budget_s):
+def cpu_baseline(wl, budget_s, kind="ags"):
     """The oracle as it stands (single-threaded C) on the host: a bounded number of
     full optimizer steps over the same parameter set."""
     pset, w, m, g = _host_inputs(wl)
-    t1 = _oracle_steps(wl, w, m, g, 1)
+    t1 = _oracle_steps(wl, w, m, g, 1, kind)
     steps = max(1, min(50, int(budget_s / max(t1, 1e-6))))
-    t = _oracle_steps(wl, w, m, g, steps)
+    t = _oracle_steps(wl, w, m, g, steps, kind)
     return {"value": pset.n_params * steps / t, "unit": UNIT, "cores": 1, "kind": "oracle",
             "sample": f"{steps} full steps of the {wl.name} parameter set "
                       f"({pset.n_params} params, {pset.n_tensors} tensors, K={wl.K}) on the host, "
@@ -256,16 +269,19 @@ def run_reference(args, wl):
     if rank != 0:
         return
     pset_full = wl.pset
+    kind = args.step_kind
+    if STEP_KINDS[kind][1] and wl.K == 1:
+        raise SystemExit("--step-kind refresh needs K > 1 (g_small is replica 0)")
     _, w, m, g = _host_inputs(wl)
-    t1 = _oracle_steps(wl, w, m, g, 1)
+    t1 = _oracle_steps(wl, w, m, g, 1, kind)
     total = args.steps + args.warmup
     frac = min(1.0, 120.0 / max(1e-9, total * t1))
     if frac < 1.0:
         pset, w, m, g = _host_inputs(wl, frac)
     else:
         pset = pset_full
-    _oracle_steps(wl, w, m, g, args.warmup)
-    t = _oracle_steps(wl, w, m, g, args.steps)
+    _oracle_steps(wl, w, m, g, args.warmup, kind)
+    t = _oracle_steps(wl, w, m, g, args.steps, kind)
     value = pset.n_params * args.steps / t
     sample = (f"each step: the single-threaded C oracle over "
               f"{'all' if frac >= 1.0 else 'the first'} {pset.n_tensors} tensors "
@@ -274,7 +290,7 @@ def run_reference(args, wl):
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * t / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-        "data": "synthetic", "config": _config(wl, pset_full),
+        "data": "synthetic", "config": _config(wl, pset_full, kind),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -282,12 +298,22 @@ def run_reference(args, wl):
     print(json.dumps(line), flush=True)
 
 
-def _config(wl, pset):
+STEP_KIND_TEXT = {
+    "ags": "Algorithm 1 step (AGS rule, per-tensor gradscale)",
+    "refresh": "Algorithm 1 step that also refreshes the gradscale (UpdateGradScale, g_small = "
+               "replica 0)",
+    "lars": "LARS rule step (coefficient 0.001 |w| / |gbar|)",
+}
+
+
+def _config(wl, pset, kind="ags"):
     return {"workload": f"{wl.name} parameter set, K={wl.K} replica gradient buffers",
+            "step": STEP_KIND_TEXT[kind],
             "params": pset.n_params, "tensors": pset.n_tensors, "K": wl.K,
             "global_batch": None, "seq_len": None, "parallelism": "replicas only (1 step per GPU)",
             "l2": "inputs larger than L2 (no flush): "
-                  f"{(4 * wl.K + 16) * pset.n_params / 1e9:.2f} GB touched per step vs 126 MB L2"}
+                  f"{step_min_bytes_per_param(wl.K, STEP_KINDS[kind][0]) * pset.n_params / 1e9:.2f}"
+                  " GB touched per step vs 126 MB L2"}
 
 
 # ---------------------------------------------------------------------------
@@ -313,12 +339,24 @@ def run_ours(args, wl):
     pset = wl.pset
     N = pset.n_params
     K = wl.K
+    kind = args.step_kind
+    read_w, refresh = STEP_KINDS[kind]
+    if refresh and K == 1:
+        raise SystemExit("--step-kind refresh needs K > 1 (g_small is replica 0)")
     buf = W.allocate(wl, "cuda")
     W.fill_state(buf, wl)
     W.fill_grads(buf, wl, step=1)
     stream = torch.cuda.Stream()
     torch.cuda.synchronize()
-    step = T.AGSOptimizerStep(buf.w, buf.g, buf.m, s_max=wl.smax)
+    # LARS with a trust coefficient of 1 moves w by about |w| each step: on one gradient reused
+    # for thousands of steps the weights overflow within ~120 steps, and every tile then takes
+    # the exact-fp64 fallback of the precise norms.  0.001 keeps them bounded.
+    step = T.AGSOptimizerStep(buf.w, buf.g, buf.m, s_max=wl.smax,
+                              rule=T.TULA_RULE_LARS if kind == "lars" else T.TULA_RULE_AGS,
+                              lars_trust=LARS_TRUST)
+
+    def one_step():
+        step.step(wl.lr, wl.momentum, wl.weight_decay, refresh_scale=refresh, stream=stream)
 
     def barrier():
         if ws > 1:
@@ -327,7 +365,8 @@ def run_ours(args, wl):
     with torch.cuda.stream(stream):
         for i in range(args.warmup):
             # the first warm-up step refreshes the gradscale (UpdateGradScale needs K > 1)
-            step.step(wl.lr, wl.momentum, wl.weight_decay, refresh_scale=(i == 0 and K > 1),
+            step.step(wl.lr, wl.momentum, wl.weight_decay,
+                      refresh_scale=refresh or (kind == "ags" and i == 0 and K > 1),
                       stream=stream)
     stream.synchronize()
 
@@ -348,7 +387,7 @@ def run_ours(args, wl):
     with torch.cuda.stream(stream):
         while time.time() - t0 < args.soak_s:
             for _ in range(20):
-                step.step(wl.lr, wl.momentum, wl.weight_decay, stream=stream)
+                one_step()
             soak += 20
             stream.synchronize()
     barrier()
@@ -358,7 +397,7 @@ def run_ours(args, wl):
     with torch.cuda.stream(stream):
         t_start.record(stream)
         for _ in range(args.steps):
-            step.step(wl.lr, wl.momentum, wl.weight_decay, stream=stream)
+            one_step()
         t_end.record(stream)
     torch.cuda.synchronize()
     barrier()
@@ -371,7 +410,7 @@ def run_ours(args, wl):
     with torch.cuda.stream(stream):
         for trio in evs:
             step.set_trace_events(trio)
-            step.step(wl.lr, wl.momentum, wl.weight_decay, stream=stream)
+            one_step()
     step.set_trace_events(None)
     torch.cuda.synchronize()
     # kernel boundaries: [0] k_reduce [1] k_combine (pass 1) [2] k_update [3] k_combine [4]
@@ -401,7 +440,7 @@ def run_ours(args, wl):
         for _ in range(args.e2e_steps):
             for k in range(K):
                 buf.g_flats[k][:buf.total].copy_(host_g[k], non_blocking=True)
-            step.step(wl.lr, wl.momentum, wl.weight_decay, stream=stream)
+            one_step()
             host_state.copy_(step.state, non_blocking=True)
             host_stats.copy_(step.stats, non_blocking=True)
         e_end.record(stream)
@@ -417,19 +456,22 @@ def run_ours(args, wl):
     peak, peak_kind = _peaks()
     p1_avg_ms = statistics.fmean(t_red)
     p2_avg_ms = statistics.fmean(t_upd)
-    p1_bytes = pass1_bytes_per_param(K) * N
+    p1_bytes = pass1_bytes_per_param(K, read_w) * N
     p2_bytes = pass2_bytes_per_param() * N
     achieved = p1_bytes / (p1_avg_ms / 1e3) / 1e9
     ms_per_step = t_max_ms / args.steps
-    step_gbs = step_min_bytes_per_param(K) * N / (ms_per_step / 1e3) / 1e9
-    traffic = _ncu_traffic("k_reduce", wl.name, N)
+    step_gbs = step_min_bytes_per_param(K, read_w) * N / (ms_per_step / 1e3) / 1e9
+    red_name = "k_reduce" if kind == "ags" else f"k_reduce_{kind}"
+    traffic = _ncu_traffic(red_name, wl.name, N)
     line = {
         "metric": METRIC, "value": job_throughput(N, args.steps, ws, t_max_ms), "unit": UNIT,
         "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
         "steps_per_s": 1e3 / ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": _config(wl, pset),
-        "roofline": {"bound": "hbm", "kernel": "k_reduce (replica mean + tile norms)",
+        "config": _config(wl, pset, kind),
+        "roofline": {"bound": "hbm",
+                     "kernel": "k_reduce (replica mean + tile norms"
+                               + (")" if kind == "ags" else ", precise norms)"),
                      "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "traffic": traffic, "bytes_per_launch": p1_bytes,
@@ -440,18 +482,19 @@ def run_ours(args, wl):
                         "frac": p2_bytes / (p2_avg_ms / 1e3) / 1e9 / peak},
         "combine_ms": {"after_reduce": statistics.fmean(t_cmb1),
                        "after_update": statistics.fmean(t_cmb2)},
-        "step_hbm": {"algorithmic_bytes_per_param": step_min_bytes_per_param(K),
+        "step_hbm": {"algorithmic_bytes_per_param": step_min_bytes_per_param(K, read_w),
                      "achieved_gbs": step_gbs, "frac": step_gbs / peak,
                      "frac_of_8tbs": step_gbs / 8000.0,
-                     "design_bytes_per_param": step_design_bytes_per_param(K),
-                     "design_gbs": step_design_bytes_per_param(K) * N / (ms_per_step / 1e3) / 1e9},
+                     "design_bytes_per_param": step_design_bytes_per_param(K, read_w),
+                     "design_gbs": step_design_bytes_per_param(K, read_w) * N
+                     / (ms_per_step / 1e3) / 1e9},
         "e2e": e2e,
         "gpu_launches": launches,
         "clocks": clocks,
         "soak_steps": soak,
     }
     if not args.no_cpu_baseline and ws == 1:
-        line["cpu_baseline"] = cpu_baseline(wl, args.cpu_sample_s)
+        line["cpu_baseline"] = cpu_baseline(wl, args.cpu_sample_s, kind)
     print(json.dumps(line), flush=True)
     if ws > 1:
         dist.destroy_process_group()

@@ -85,6 +85,7 @@ constexpr int kCombWarps = 4;           // k_combine: one warp per segment, 4 pe
 constexpr int kSegTiles = 256;          // tile partials per combine segment (8 per lane)
 constexpr int kParamBudget = 31 * 1024; // kernel parameter bytes per launch (limit 32764)
 constexpr int kAcc = 3;                 // partial sums per pass-1 tile: |gbar|^2, |g_0|^2, |w|^2
+constexpr int kPrecCols = 1;            // float4 columns per step of the precise path's tile loop
 constexpr int kTsum = 4;                // per-tensor sums (stride)
 constexpr unsigned kFull = 0xffffffffu;
 constexpr uint32_t kSpinLimit = 1u << 19;  // bound on every mbarrier wait (~2 s on GB300)
@@ -191,17 +192,6 @@ __device__ __forceinline__ float sq4(float acc, float4 v) {
     return acc;
 }
 
-// fp64 sum of exact squares (an fp32 square is exact in fp64), one DFMA per term
-// Precise sum of squares: each square is exact in fp64 and rounded once into
-// the running sum (this path is bound by GB300's FP64 throughput, not latency).
-__device__ __forceinline__ double dsq4(double acc, float4 v) {
-    acc = __fma_rn((double)v.x, (double)v.x, acc);
-    acc = __fma_rn((double)v.y, (double)v.y, acc);
-    acc = __fma_rn((double)v.z, (double)v.z, acc);
-    acc = __fma_rn((double)v.w, (double)v.w, acc);
-    return acc;
-}
-
 __device__ __forceinline__ float4 add4(float4 a, float4 b) {
     return make_float4(__fadd_rn(a.x, b.x), __fadd_rn(a.y, b.y), __fadd_rn(a.z, b.z),
                        __fadd_rn(a.w, b.w));
@@ -273,6 +263,48 @@ __device__ __forceinline__ float2 ff_add(float2 a, float2 b) {
 __device__ __forceinline__ double ff_to_double(float2 v) {
     return __dadd_rn((double)v.x, (double)v.y);
 }
+
+// Precise sums of squares on the FP32 pipes.  x*x == p + e exactly, with
+// p = fl(x*x) and e = fma(x, x, -p), unless p overflows or e underflows.  p
+// joins the running high part by TwoSum, both error terms join the low part,
+// and Fast2Sum renormalises the pair, so each addition errs by at most ~2u^2 of
+// the running sum (u = 2^-24) with no fp64 instruction; one pair per float4
+// component keeps four independent chains in flight.  The streaming loop has no
+// range test (a branch there would cost more than the arithmetic): an overflow
+// shows as a non-finite pair, and an underflowed e errs by at most 2^-149, so a
+// lane sum of at least 2^-77 is as good as exact; dw_lane_ok tests both once
+// per tile, and the tile is redone in fp64 when a lane fails.
+struct Dw4 {
+    float hi[4], lo[4];
+};
+__device__ __forceinline__ void dw_zero(Dw4 &a) {
+#pragma unroll
+    for (int c = 0; c < 4; ++c) a.hi[c] = a.lo[c] = 0.f;
+}
+__device__ __forceinline__ void dw_sq(float &hi, float &lo, float x) {
+    const float p = __fmul_rn(x, x);
+    const float e = __fmaf_rn(x, x, -p);
+    const float2 t = two_sum(hi, p);
+    const float l = __fadd_rn(lo, __fadd_rn(t.y, e));
+    hi = __fadd_rn(t.x, l);
+    lo = __fsub_rn(l, __fsub_rn(hi, t.x));
+}
+__device__ __forceinline__ void dw_sq4(Dw4 &a, float4 v) {
+    dw_sq(a.hi[0], a.lo[0], v.x);
+    dw_sq(a.hi[1], a.lo[1], v.y);
+    dw_sq(a.hi[2], a.lo[2], v.z);
+    dw_sq(a.hi[3], a.lo[3], v.w);
+}
+// The four pairs added in a fixed tree.
+__device__ __forceinline__ float2 dw_pair(const Dw4 &a) {
+    const float2 c01 = ff_add(make_float2(a.hi[0], a.lo[0]), make_float2(a.hi[1], a.lo[1]));
+    const float2 c23 = ff_add(make_float2(a.hi[2], a.lo[2]), make_float2(a.hi[3], a.lo[3]));
+    return ff_add(c01, c23);
+}
+__device__ __forceinline__ bool dw_lane_ok(float2 v) {
+    return v.x >= 0x1p-77f && v.x <= 3.0e38f;  // false for 0, tiny sums, inf and NaN
+}
+
 // Partial sums travel as float-float pairs, or as fp64 where the norms feed a
 // coefficient (precise mode): Part<P>::T is the stored type, zero/add/tree work
 // on it.  Both are 8 bytes, so the workspace layout is the same.
@@ -640,12 +672,14 @@ __device__ __forceinline__ void ring_setup(unsigned char *smem, uint64_t *&full,
 }
 
 // A consumer's wait for its j-th tile: the launch tile index, -1 when no tile
-// is left, -2 when the wait ran out (reported).
+// is left, -2 when the wait ran out (reported).  Called by the whole warp; the
+// result is the same in every lane (a lane whose bounded wait ran out makes
+// the warp stop), so the warp stays converged for its shuffles and votes.
 template <typename R>
 __device__ __forceinline__ int next_tile(const Scalars &sc, int j, uint64_t *full,
                                          const int *stage_tile) {
     const int s = j % R::kStages;
-    if (!mbar_wait(&full[s], (uint32_t)((j / R::kStages) & 1))) {
+    if (!__all_sync(kFull, mbar_wait(&full[s], (uint32_t)((j / R::kStages) & 1)))) {
         if ((threadIdx.x & 31) == 0) report_timeout(sc);
         return -2;
     }
@@ -659,9 +693,10 @@ __device__ __forceinline__ int next_tile(const Scalars &sc, int j, uint64_t *ful
 // Template: KT = replicas known at compile time (0: runtime K <= 16);
 // WM = write the mean over replica 0; RW = also reduce |w|^2;
 // SS = g_small is a separate stream instead of replica 0;
-// PR = precise norms: every exact fp64 square is added in fp64, and the tile's
-// lanes in an fp64 tree (relative error ~1e-15), for norms that feed a
-// per-tensor coefficient (UpdateGradScale, LARS).  Otherwise the tile's sum
+// PR = precise norms: every square is split exactly into two fp32 parts and
+// added as a float-float pair (Dw4), each lane's pairs go to fp64 once per tile,
+// and the tile's lanes are added in an fp64 tree (relative error ~1e-14), for
+// norms that feed a per-tensor coefficient (UpdateGradScale, LARS).  Otherwise the tile's sum
 // stays in fp32: each lane adds <= 16 squares per group of 4 columns, then the
 // group sums, then a 5-level tree across lanes, a relative error below 71 ulp
 // (4e-6) of the tile's sum; tiles are combined in fp64.  That is what the
@@ -679,23 +714,59 @@ struct P1 {
 // One float4 column of a tile: mean, squares.  x0 = replica 0, s = sum.
 template <int KT, bool WM, bool RW, bool SS, bool PR>
 __device__ __forceinline__ void column1(float4 x0, float4 s, float4 wv, float4 sv, float *out,
-                                        const Scalars &sc, int K, double &ag, double &as,
-                                        double &aw, float &pg, float &ps, float &pw) {
+                                        const Scalars &sc, int K, Dw4 &ag, Dw4 &as, Dw4 &aw,
+                                        float &pg, float &ps, float &pw) {
     if (K > 1) {
         s = mean4<KT>(s, sc);
         if (WM) st_keep(out, s);
     }
     if (PR) {
-        ag = dsq4(ag, s);
-        if (K > 1) as = dsq4(as, x0);
-        if (SS) as = dsq4(as, sv);
-        if (RW) aw = dsq4(aw, wv);
+        dw_sq4(ag, s);
+        if (K > 1) dw_sq4(as, x0);
+        if (SS) dw_sq4(as, sv);
+        if (RW) dw_sq4(aw, wv);
     } else {
         pg = sq4(pg, s);
         if (K > 1) ps = sq4(ps, x0);
         if (SS) ps = sq4(ps, sv);
         if (RW) pw = sq4(pw, wv);
     }
+}
+
+// A tile's shared-memory columns again, every square exact in fp64 and added
+// in fp64: the precise path's fallback when a lane's float-float sum is not
+// finite or too small to hold its error (dw_lane_ok).  Out of line, so that
+// the streaming loop keeps its shape.
+struct D3 {
+    double g, s, w;
+};
+template <int KT, bool RW, bool SS>
+__device__ __noinline__ D3 tile_cols_fp64(uint32_t stage, int chunk, int nv, const Scalars &sc) {
+    const int lane = threadIdx.x & 31;
+    const int K = KT > 0 ? KT : sc.K;
+    const uint32_t sw_s = stage + (uint32_t)(K * chunk * 4);
+    const uint32_t ss_s = stage + (uint32_t)((K + (RW ? 1 : 0)) * chunk * 4);
+    D3 r = {0.0, 0.0, 0.0};
+    for (int v = lane; v < nv; v += 32) {
+        const float4 x0 = lds4(stage + (uint32_t)(16 * v));
+        float4 s = x0;
+        for (int k = 1; k < K; ++k) s = add4(s, lds4(stage + (uint32_t)((k * chunk + 4 * v) * 4)));
+        if (K > 1) s = mean4<KT>(s, sc);
+        const float gs[4] = {s.x, s.y, s.z, s.w};
+        const float g0[4] = {x0.x, x0.y, x0.z, x0.w};
+        float4 wv = make_float4(0.f, 0.f, 0.f, 0.f), sv = wv;
+        if (RW) wv = lds4(sw_s + (uint32_t)(16 * v));
+        if (SS) sv = lds4(ss_s + (uint32_t)(16 * v));
+        const float ws[4] = {wv.x, wv.y, wv.z, wv.w};
+        const float ss[4] = {sv.x, sv.y, sv.z, sv.w};
+        for (int c = 0; c < 4; ++c) {
+            r.g = __fma_rn((double)gs[c], (double)gs[c], r.g);
+            if (K > 1) r.s = __fma_rn((double)g0[c], (double)g0[c], r.s);
+            if (SS) r.s = __fma_rn((double)ss[c], (double)ss[c], r.s);
+            if (RW) r.w = __fma_rn((double)ws[c], (double)ws[c], r.w);
+        }
+    }
+    return r;
 }
 
 // Per-lane partial sums of one tile (not yet reduced across the warp).
@@ -709,7 +780,12 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
     const uint32_t sw_s = stage + (uint32_t)(K * chunk * 4);
     const uint32_t ss_s = stage + (uint32_t)((K + (RW ? 1 : 0)) * chunk * 4);
     float *out = const_cast<float *>(ptr[0]) + q.begin;
-    double ag = 0.0, as = 0.0, aw = 0.0;  // precise (PR) sums
+    Dw4 ag, as, aw;                       // precise (PR) sums of the shared-memory columns
+    dw_zero(ag);
+    dw_zero(as);
+    dw_zero(aw);
+    double rg = 0.0, rs = 0.0, rw = 0.0;  // precise (PR) sums of the elements loaded directly
+    const int ncols = nv;                 // the shared-memory columns (nv is reused below)
     float fg = 0.f, fs = 0.f, fw = 0.f;   // fp32 sums (not PR)
 
     if constexpr (KT > 0) {
@@ -717,11 +793,15 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
         constexpr int COLS = CH / 128;  // float4 columns per lane of a full tile
         if (nv == CH / 4) {
             // Full tile: every lane has COLS columns; all loads of a column issue together.
-#pragma unroll
-            for (int c0 = 0; c0 < COLS; c0 += 4) {
+            // The precise path walks them kPrecCols at a time in a rolled loop: unrolled, its
+            // float-float arithmetic outgrows the instruction cache.
+            constexpr int G = PR ? kPrecCols : 4;
+            constexpr int UNR = PR ? 1 : (COLS + 3) / 4;
+#pragma unroll UNR
+            for (int c0 = 0; c0 < COLS; c0 += G) {
                 float pg = 0.f, ps = 0.f, pw = 0.f;
 #pragma unroll
-                for (int u = 0; u < 4; ++u) {
+                for (int u = 0; u < G; ++u) {
                     if (c0 + u < COLS) {
                         const int v = lane + 32 * (c0 + u);
                         float4 x[KT];
@@ -780,10 +860,10 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
             const float y_s = SS ? __ldcs(ptr[KS + 1] + j) : 0.f;
             const float y_w = RW ? __ldcs(ptr[KS] + j) : 0.f;
             if (PR) {
-                if (K > 1) as = __fma_rn((double)x0, (double)x0, as);
-                ag = __fma_rn((double)s, (double)s, ag);
-                if (SS) as = __fma_rn((double)y_s, (double)y_s, as);
-                if (RW) aw = __fma_rn((double)y_w, (double)y_w, aw);
+                if (K > 1) rs = __fma_rn((double)x0, (double)x0, rs);
+                rg = __fma_rn((double)s, (double)s, rg);
+                if (SS) rs = __fma_rn((double)y_s, (double)y_s, rs);
+                if (RW) rw = __fma_rn((double)y_w, (double)y_w, rw);
             } else {
                 if (K > 1) fs = __fmaf_rn(x0, x0, fs);
                 fg = __fmaf_rn(s, s, fg);
@@ -793,9 +873,24 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
         }
     }
     if (PR) {
-        accd[0] = ag;
-        accd[1] = (K > 1 || SS) ? as : ag;  // K = 1: replica 0 is the mean
-        accd[2] = aw;
+        // The warp is converged again here (the loops above end in every lane).
+        const float2 pg = dw_pair(ag), ps = dw_pair(as), pw = dw_pair(aw);
+        const bool bad = lane < ncols && !(dw_lane_ok(pg) && (!(K > 1 || SS) || dw_lane_ok(ps)) &&
+                                           (!RW || dw_lane_ok(pw)));
+        double cg, cs, cw;
+        if (__any_sync(kFull, bad)) {
+            const D3 f = tile_cols_fp64<KT, RW, SS>(stage, chunk, ncols, sc);
+            cg = f.g;
+            cs = f.s;
+            cw = f.w;
+        } else {
+            cg = ff_to_double(pg);
+            cs = ff_to_double(ps);
+            cw = ff_to_double(pw);
+        }
+        accd[0] = __dadd_rn(cg, rg);
+        accd[1] = (K > 1 || SS) ? __dadd_rn(cs, rs) : accd[0];  // K = 1: replica 0 is the mean
+        accd[2] = RW ? __dadd_rn(cw, rw) : 0.0;
     } else {
         accf[0] = fg;
         accf[1] = (K > 1 || SS) ? fs : fg;

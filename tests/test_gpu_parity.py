@@ -411,3 +411,54 @@ def test_calls_back_to_back_on_one_workspace_and_stream(K):
         assert np.array_equal(buf.g[0][p].reshape(-1).cpu().numpy(), g_h[0][p]), p
         assert_f32_close(buf.w[p].reshape(-1).cpu().numpy(), pair.w_h[p], f"w[{p}]")
         assert_f32_close(buf.m[p].reshape(-1).cpu().numpy(), pair.m_h[p], f"m[{p}]")
+
+
+def _extreme_pset(streams):
+    """Tensors of one element to several tiles (ragged tails) of a pass-1 tile of `streams`
+    streams, three times over, for per-tensor gradient factors spread over 46 decades."""
+    ps = W.ParamSet("extremes")
+    t = T.tula_ags_chunk_elems(1, streams)
+    for _ in range(3):
+        for n in (1, 5, 64, 1000, t - 1, t + 3, 2 * t + 7, 40000):
+            ps.add((n,), W.KIND_NORMAL)
+    return ps
+
+
+def _extreme_workload(seed, ps):
+    wl = W.workload("stress_k4", seed=seed, factor_range=(1e-24, 1e22), zero_patterns=False)
+    f = W._factors(wl, ps)
+    # squares below fp32's normal range, beyond its largest value, and ordinary ones
+    assert (f < 1e-20).any() and (f > 1e20).any() and ((f > 1e-3) & (f < 1e3)).any()
+    return wl
+
+
+def test_lars_steps_over_the_whole_float_range():
+    """LARS steps take every pass-1 norm precisely.  Gradient factors from 1e-24 to 1e22: the
+    squares of some tensors underflow or overflow fp32 (they go through fp64), the others are
+    split exactly into float-float pairs; coefficients, norms and updates match the oracle."""
+    ps = _extreme_pset(3)
+    wl = _extreme_workload(97, ps)
+    pair = Pair(wl, K=2, pset=ps, rule=T.TULA_RULE_LARS, lars_trust=0.01)
+    pair.step(1, 1.0)
+    pair.step(2, 1.0)
+
+
+def test_update_scale_over_the_whole_float_range():
+    """UpdateGradScale per tensor (precise norms of g_small and g_large) over the same range,
+    with s_max out of the way: each scale within 2 ulp of the oracle's fp64 ratio."""
+    ps = _extreme_pset(2)
+    wl = _extreme_workload(105, ps)
+    buf = W.allocate(wl, "cuda", K=2, pset=ps)
+    W.fill_grads(buf, wl, step=1)
+    gs, gl = buf.g[1], buf.g[0]
+    n = buf.pset.n_tensors
+    hp = T.tula_ags_default_hparams(2)
+    hp.s_max = 1e30
+    scale = torch.zeros(n, dtype=torch.float32, device="cuda")
+    ws = T.new_workspace(buf.numels, 1)
+    hp.scale, hp.workspace, hp.workspace_bytes = scale.data_ptr(), ws.data_ptr(), ws.numel()
+    T.tula_ags_update_scale(gs, gl, hp)
+    ref = np.zeros(n, np.float32)
+    O.update_scale(W.to_numpy(gs), W.to_numpy(gl), hp.eps, 1e30, O.GRAN_TENSOR, scale=ref)
+    torch.cuda.synchronize()
+    assert_norm_close(scale.cpu().numpy(), ref, "scale", rtol=2.0 ** -22)
