@@ -793,11 +793,11 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
         constexpr int COLS = CH / 128;  // float4 columns per lane of a full tile
         if (nv == CH / 4) {
             // Full tile: every lane has COLS columns; all loads of a column issue together.
-            // The precise path walks them kPrecCols at a time in a rolled loop: unrolled, its
-            // float-float arithmetic outgrows the instruction cache.
+            // The loop over groups of G columns stays rolled: unrolled over the tile (and
+            // again for each of the kPend tiles), the body outgrows the instruction cache.
+            // The precise path's float-float arithmetic takes kPrecCols columns per group.
             constexpr int G = PR ? kPrecCols : 4;
-            constexpr int UNR = PR ? 1 : (COLS + 3) / 4;
-#pragma unroll UNR
+#pragma unroll 1
             for (int c0 = 0; c0 < COLS; c0 += G) {
                 float pg = 0.f, ps = 0.f, pw = 0.f;
 #pragma unroll
@@ -1348,11 +1348,13 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
             const float4 cdef = PE ? make_float4(1.f, 1.f, 1.f, 1.f) : make_float4(ct, ct, ct, ct);
             float aw = 0.f;  // fp32 |w|^2 of the tile (statistics only)
             if (nv == CH / 4) {
-#pragma unroll
-                for (int c0 = 0; c0 < COLS; c0 += 4) {
+                // Two columns per step of a rolled loop (unrolled over the tile, the body
+                // outgrew the instruction cache: 82.5 -> 75.5 us per ResNet-50 update pass).
+#pragma unroll 1
+                for (int c0 = 0; c0 < COLS; c0 += 2) {
                     float pw = 0.f;
 #pragma unroll
-                    for (int u = 0; u < 4; ++u) {
+                    for (int u = 0; u < 2; ++u) {
                         if (c0 + u < COLS) {
                             const int v = lane + 32 * (c0 + u);
                             const float4 g4 = lds4(stage + (uint32_t)(16 * v));
