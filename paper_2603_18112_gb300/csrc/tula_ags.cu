@@ -48,6 +48,7 @@
 #include <cstring>
 #include <memory>
 #include <mutex>
+#include <type_traits>
 #include <utility>
 #include <vector>
 
@@ -76,6 +77,13 @@ struct Ring {
 // consumers.  Pass 2 does ~11 flops per element over 3-4 streams: its
 // consumers, not HBM, set the pace with three warps, so it runs four.
 using Ring1 = Ring<32, 6, 3>;
+// The precise pass 1 (float-float squares) spends ~13 dependent FP32 instructions per element
+// and norm: six consumers, two per scheduler, hide that latency.  Same stages, same tiles.
+using Ring1P = Ring<32, 6, 6>;
+template <bool PR>
+using Ring1For = std::conditional_t<PR, Ring1P, Ring1>;
+static_assert(Ring1P::kStageBytes == Ring1::kStageBytes && Ring1P::kStages == Ring1::kStages,
+              "both pass-1 rings cut the same tiles");
 using Ring2 = Ring<24, 8, 4>;
 constexpr int kDynTiles = 64;            // tiles per CTA from which a launch claims its tiles
 constexpr unsigned kClaim = 4;           // tiles per claim
@@ -899,7 +907,7 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
 }
 
 template <int KT, bool WM, bool RW, bool SS, bool PR>
-__global__ void __launch_bounds__(Ring1::kThreads, 1)
+__global__ void __launch_bounds__(Ring1For<PR>::kThreads, 1)
     k_reduce(const __grid_constant__ Table<P1<KT>::NP> tab, const __grid_constant__ Scalars sc) {
     constexpr int KS = P1<KT>::KS;
     constexpr int NSMAX = KS + 2;
@@ -918,7 +926,8 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
     if (!early) grid_wait();
     uint64_t *full, *empty;
     int *stage_tile;
-    ring_setup<Ring1>(smem, full, empty, stage_tile);
+    using R1 = Ring1For<PR>;
+    ring_setup<R1>(smem, full, empty, stage_tile);
     const int js = static_tiles(tab.nc);
     const uint32_t ring = smem_addr(smem);
     const int warp = threadIdx.x >> 5;
@@ -931,7 +940,7 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
     if (RW) roles[ns++] = KS;
     if (SS) roles[ns++] = KS + 1;
     if (warp == 0) {
-        produce<Ring1, P1<KT>::NP, NSMAX>(tab, sc, roles, ns, chunk, js, sc.tiles, ring, full,
+        produce<R1, P1<KT>::NP, NSMAX>(tab, sc, roles, ns, chunk, js, sc.tiles, ring, full,
                                           empty, stage_tile);
         return;
     }
@@ -940,13 +949,13 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
     const int cw = warp - 1;
     TensorCache tc;
     bool stop = false;
-    for (int jb = cw; !stop; jb += Ring1::kConsumers * kPend) {
+    for (int jb = cw; !stop; jb += R1::kConsumers * kPend) {
         double pendd[PR ? kPend * kAcc : 1];
         float pendf[PR ? 1 : kPend * kAcc];
         int ptile[kPend];
 #pragma unroll
         for (int p = 0; p < kPend; ++p) {
-            const int j = jb + p * Ring1::kConsumers;
+            const int j = jb + p * R1::kConsumers;
             ptile[p] = -1;
 #pragma unroll
             for (int a = 0; a < kAcc; ++a) {
@@ -958,7 +967,7 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
             int c = j < js ? static_tile(j) : -1;
             TilePos q;
             if (c >= 0) q = tc.at(tab, c, chunk, my_role, ns);
-            const int got = next_tile<Ring1>(sc, j, full, stage_tile);
+            const int got = next_tile<R1>(sc, j, full, stage_tile);
             if (got < 0) {
                 stop = true;
                 continue;
@@ -967,11 +976,11 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
                 c = got;
                 q = tc.at(tab, c, chunk, my_role, ns);
             }
-            const int s = j % Ring1::kStages;
+            const int s = j % R1::kStages;
             const float *const *ptr = tab.ptr[q.t];
             double accd[kAcc];
             float accf[kAcc];
-            reduce_tile<KT, WM, RW, SS, PR>(ring + (uint32_t)s * Ring1::kStageBytes, chunk, ptr, q,
+            reduce_tile<KT, WM, RW, SS, PR>(ring + (uint32_t)s * R1::kStageBytes, chunk, ptr, q,
                                             tc.nv, sc, accd, accf);
             __syncwarp();
             if (lane == 0) mbar_arrive(&empty[s]);
@@ -1747,8 +1756,8 @@ int run_reduce_k(int K, int n, const int64_t *numels, const Scalars &sc, int gri
                  Fill fill, void *mid_event) {
     const int chunk = chunk1(K, RW, SS);
     int rc = launch_streaming<P1<KT>::NP>(k_reduce<KT, WM, RW, SS, PR>, n, numels, chunk,
-                                          Ring1::kThreads, Ring1::kSmemBytes, sc, grid, s,
-                                          fill);
+                                          Ring1For<PR>::kThreads, Ring1For<PR>::kSmemBytes, sc,
+                                          grid, s, fill);
     if (rc) return rc;
     record(mid_event, s);
     return launch_combine<kAcc, PR>(n, numels, chunk, sc, s);
