@@ -115,7 +115,10 @@ typedef struct tula_ags_hparams {
     float eps;         /* stability term of UpdateGradScale (default 1e-8, Algorithm 1) */
     float s_max;       /* bound on gradscale, sqrt(b_large / b_small) (default sqrt(K)) */
     float static_s;    /* s of Eq. 8 for TULA_RULE_STATIC (default 1) */
-    float lars_trust;  /* trust coefficient for TULA_RULE_LARS (default 1) */
+    float lars_trust;  /* trust coefficient for TULA_RULE_LARS (default 1).  c_p is about
+                          lars_trust * |w_p| / |gbar_p|, so a step moves w by roughly
+                          lr * lars_trust * |w| / (1 - momentum): with lr 0.1 and momentum 0.9,
+                          a trust of 1 doubles |w| per step.  Values near 1e-3 keep it small. */
     float *scale;                 /* device fp32 [n_tensors]: gradscale per tensor (AGS, PER_TENSOR);
                                      written when refresh_scale is set */
     float *const *scale_elem;     /* HOST array of n_tensors device fp32 pointers: gradscale per
