@@ -25,3 +25,31 @@ def test_step_kinds():
     assert bench.STEP_KINDS == {"ags": (False, False), "refresh": (False, True),
                                 "lars": (True, False)}
     assert set(bench.STEP_KIND_TEXT) == set(bench.STEP_KINDS)
+
+
+@pytest.mark.parametrize("kind", ["ags", "lars"])
+def test_reference_arm_prints_the_contract_line(kind):
+    """`bench.py --impl reference` (the oracle on the host) prints one JSON line with the keys
+    the benchmark contract asks for, on the same metric and unit as the GPU arm."""
+    import json
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    out = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--impl", "reference",
+                          "--workload", "resnet20", "--steps", "1", "--warmup", "0",
+                          "--step-kind", kind],
+                         capture_output=True, text=True, timeout=300, cwd=root)
+    assert out.returncode == 0, out.stderr[-2000:]
+    lines = [ln for ln in out.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["unit"] == bench.UNIT
+    assert d["value"] > 0 and d["higher_is_better"] is True and d["n_gpus"] == 1
+    assert d["steps"] == 1 and d["warmup"] == 0 and d["vs_baseline"] is None
+    assert d["config"]["workload"].startswith("resnet20")
+    assert d["config"]["step"] == bench.STEP_KIND_TEXT[kind]
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
+    assert d["e2e"] == {"value": d["value"], "unit": bench.UNIT, "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}
