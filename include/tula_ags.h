@@ -97,7 +97,8 @@ extern "C" {
 #define TULA_STAT_G0_SQ 2     /* |g_{0,p}|^2, replica 0 before averaging */
 #define TULA_STAT_W_NORM 3    /* |w_p| */
 #define TULA_STAT_G_NORM 4    /* |gbar_p| */
-#define TULA_STAT_RATIO 5     /* |w_p| / |gbar_p| (LARS trust ratio), 0 when |gbar_p| = 0 */
+#define TULA_STAT_RATIO 5     /* |w_p| / |gbar_p|: the per-layer ratio LARS scales the learning
+                                 rate by (Sec. V-B); 0 when |gbar_p| = 0 */
 #define TULA_STAT_COEF 6      /* c_p applied to the gradient this step (NaN: per-element scale) */
 #define TULA_STAT_SCALE 7     /* gradscale_p after the step (0 without a per-tensor scale) */
 #define TULA_STATS_LEN 8
@@ -174,6 +175,11 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
  * Per-layer statistics without an update (read-only on every tensor): rows of
  * TULA_STATS_LEN fp64 as above, columns TULA_STAT_COEF and TULA_STAT_SCALE set to 0.
  * grad_ptrs[k*n + p] as in tula_ags_step.  stats_out: device fp64 [n_tensors][8].
+ * Paper: TulaOptimizer wraps the training optimizer and tracks the gradient norm of every
+ * parameter tensor (Sec. IV-A); the squared norms of the mean gradient are the per-layer terms
+ * of |G|^2 in Eq. 5, those of replica 0 (a small-batch gradient at the same weights) are the
+ * small-batch norms of Algorithm 1's UpdateGradScale, and |w_p| / |gbar_p| is the per-layer ratio
+ * by which LARS scales the learning rate (Sec. V-B).
  */
 int tula_layer_stats(const float *const *param_ptrs, const float *const *grad_ptrs, int K,
                      const int64_t *numels, int n_tensors, double *stats_out, void *workspace,
@@ -210,19 +216,42 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
  * tensors holding up to ~1.2e9 parameters at K <= 2, ~5.1e8 at K = 8, ~2.4e8 at K = 16.  A larger
  * list is rejected with TULA_ERR_SCRATCH_LIMIT before anything is enqueued.
  *
- * Set-up: the first call on each device, with that device current, looks up the array's device
- * address (cudaGetSymbolAddress); make that first call before any stream capture.
+ * Set-up: every call looks up the array's device address in the current device's context
+ * (cudaGetSymbolAddress, a host-side lookup), so the address never goes stale, also after
+ * cudaDeviceReset.  The first call on a device also loads the library's device code there: make
+ * it, with that device current, before any stream capture.
  * Sharing: every call on a device uses the same array.  Each call clears the counters it needs
- * zeroed (an asynchronous memset on `stream`) and otherwise overwrites what the previous call
- * left, so calls that overlap on the GPU (different streams, or different host threads) race
- * and must not be issued.  Allocates nothing: no cudaMalloc, no cudaFree, no allocating library
- * call.  Arguments, semantics and other status codes are those of tula_ags_step.
+ * zeroed (two asynchronous memsets on `stream`, enqueued only once every argument has been
+ * accepted) and otherwise overwrites what the previous call left, so calls that overlap on the
+ * GPU (different streams, or different host threads) race and must not be issued.  Allocates
+ * nothing: no cudaMalloc, no cudaFree, no allocating library call.
+ * Errors: as tula_ags_step, plus TULA_ERR_SCRATCH_LIMIT.  A bounded wait that runs out inside a
+ * kernel sets the array's error word, which no later call clears: read it (and clear it) with
+ * tula_ags_static_scratch_error.  While it is set, the steps since it was last read are not
+ * valid.
  */
 #define TULA_STATIC_SCRATCH_BYTES (16u << 20)
 int tula_ags_step_static_scratch(float *const *param_ptrs, float *const *grad_ptrs,
                                  float *const *mom_ptrs, const int64_t *numels, int n_tensors,
                                  float lr, float momentum, float weight_decay,
                                  const tula_ags_hparams *hp, void *stream);
+
+/*
+ * The error word of the static scratch on the current device, read after the work already
+ * enqueued on `stream` (the call waits for that stream), then cleared: *error_out = 0 when every
+ * bounded wait of the static-scratch steps since the last read completed, bit 0 set when one ran
+ * out.  The counterpart of tula_ags_workspace_error for tula_ags_step_static_scratch (no
+ * counterpart in the paper).  TULA_ERR_ARG when error_out is NULL; TULA_ERR_CUDA when a CUDA
+ * call fails.
+ */
+int tula_ags_static_scratch_error(void *stream, int *error_out);
+
+/*
+ * Failure-detection check on the static scratch: as tula_ags_check_wait_timeout, with the error
+ * word of the static array on the current device in place of a workspace's.  Asynchronous on
+ * `stream`; about two seconds of GPU time.  No counterpart in the paper.
+ */
+int tula_ags_static_scratch_check_wait_timeout(void *stream);
 
 /* Human-readable text for a TULA_* status code. */
 const char *tula_ags_error_string(int code);

@@ -136,7 +136,8 @@ def replica_mean(grads: list[np.ndarray]) -> np.ndarray:
 
 
 def sqnorm(x: np.ndarray) -> float:
-    """|x|^2 in fp64, sequential."""
+    """|x|^2 in fp64: exact fp64 squares added from element 0 on with Neumaier's compensated
+    summation (within about 1e-16 of the exact sum)."""
     x = np.ascontiguousarray(x, dtype=np.float32)
     return _load().oracle_sqnorm(_fp(x), x.size)
 

@@ -14,7 +14,14 @@ LIB = HERE / "libtula_ags.so"
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", "-shared",
-              "-cudart", "shared", "-fmad=false", "-Xlinker", "-rpath=/usr/local/cuda/lib64"]
+              "-cudart", "shared", "-fmad=false"]
+
+
+def cuda_lib_dir(nvcc: str) -> str:
+    """The toolkit's library directory (CUDA_HOME/lib64, else next to nvcc's bin/): the shared
+    CUDA runtime the library links is found there at run time."""
+    home = os.environ.get("CUDA_HOME") or os.path.dirname(os.path.dirname(os.path.realpath(nvcc)))
+    return os.path.join(home, "lib64")
 
 
 def nvcc_path() -> str:
@@ -37,7 +44,9 @@ def build(force: bool = False, verbose: bool = False) -> Path:
     if not force and not _stale():
         return LIB
     tmp = LIB.with_name(f"{LIB.name}.{os.getpid()}.tmp")
-    cmd = [nvcc_path(), *ARCH, *NVCC_FLAGS, "-I", str(ROOT / "include"), str(SRC), "-o", str(tmp)]
+    nvcc = nvcc_path()
+    cmd = [nvcc, *ARCH, *NVCC_FLAGS, "-Xlinker", f"-rpath={cuda_lib_dir(nvcc)}",
+           "-I", str(ROOT / "include"), str(SRC), "-o", str(tmp)]
     if verbose:
         cmd.insert(1, "-Xptxas=-v")
     subprocess.run(cmd, check=True)

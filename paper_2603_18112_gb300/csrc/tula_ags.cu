@@ -1869,11 +1869,16 @@ int tula_ags_workspace_error(const void *workspace, size_t workspace_bytes,
     return TULA_OK;
 }
 
-int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mom_ptrs,
-                  const int64_t *numels, int n_tensors, float lr, float momentum,
-                  float weight_decay, const tula_ags_hparams *hp, void *stream) {
-    Plan pl;
-    if (!hp || !param_ptrs || !grad_ptrs || !valid_numels(numels, n_tensors, hp->K, &pl))
+}  // extern "C"
+
+namespace {
+
+// Every host-side check of a step's arguments except the workspace: TULA_OK or the status
+// tula_ags_step returns.  Nothing is enqueued before it passes.
+int check_step_args(float *const *param_ptrs, float *const *grad_ptrs, float *const *mom_ptrs,
+                    const int64_t *numels, int n_tensors, float momentum,
+                    const tula_ags_hparams *hp, Plan *pl) {
+    if (!hp || !param_ptrs || !grad_ptrs || !valid_numels(numels, n_tensors, hp->K, pl))
         return TULA_ERR_ARG;
     const int K = hp->K, n = n_tensors;
     if (hp->rule < TULA_RULE_AGS || hp->rule > TULA_RULE_STATIC) return TULA_ERR_ARG;
@@ -1900,12 +1905,20 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
             if (!g || !aligned4(g)) return TULA_ERR_ARG;
         }
     }
-    int rc = check_ws(hp->workspace, hp->workspace_bytes, n, pl);
-    if (rc) return rc;
+    return TULA_OK;
+}
 
+// The step's launches, once its arguments (check_step_args) and its scratch `ws` (the caller's
+// workspace or the static array) have been accepted.
+int run_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mom_ptrs,
+             const int64_t *numels, int n, float lr, float momentum, float weight_decay,
+             const tula_ags_hparams *hp, void *ws, const Plan &pl, void *stream) {
+    const int K = hp->K;
+    const bool per_elem = hp->rule == TULA_RULE_AGS && hp->granularity == TULA_SCALE_PER_ELEMENT;
+    int rc = TULA_OK;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const WsLayout L = ws_layout(n, pl);
-    Scalars sc = make_scalars(hp, K, n, hp->workspace, L, kModeStep);
+    Scalars sc = make_scalars(hp, K, n, ws, L, kModeStep);
     const bool lars = hp->rule == TULA_RULE_LARS;
     sc.read_w = lars ? 1 : 0;
     // When the mean fits in L2, every bulk load is marked to leave L2 first, so
@@ -1966,6 +1979,22 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
     if (rc) return rc;
     record(hp->trace_events[4], s);
     return TULA_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mom_ptrs,
+                  const int64_t *numels, int n_tensors, float lr, float momentum,
+                  float weight_decay, const tula_ags_hparams *hp, void *stream) {
+    Plan pl;
+    int rc = check_step_args(param_ptrs, grad_ptrs, mom_ptrs, numels, n_tensors, momentum, hp, &pl);
+    if (rc) return rc;
+    rc = check_ws(hp->workspace, hp->workspace_bytes, n_tensors, pl);
+    if (rc) return rc;
+    return run_step(param_ptrs, grad_ptrs, mom_ptrs, numels, n_tensors, lr, momentum,
+                    weight_decay, hp, hp->workspace, pl, stream);
 }
 
 int tula_layer_stats(const float *const *param_ptrs, const float *const *grad_ptrs, int K,
@@ -2067,40 +2096,36 @@ uint64_t tula_ags_launch_count(void) { return g_launches.load(std::memory_order_
 // Allocation-free step: the scratch in a static device array
 // ============================================================================
 // For callers that cannot allocate device memory (see the header).  The step
-// itself is tula_ags_step; only where its scratch lives differs.
+// itself is tula_ags_step's; only where its scratch lives differs.
 
 namespace {
 
 constexpr size_t kStaticScratchBytes = TULA_STATIC_SCRATCH_BYTES;
-constexpr int kMaxDevices = 64;
 
 // One copy per device, alive until the process exits.  In host code this name
 // is only a handle: its device address comes from cudaGetSymbolAddress.
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
 
-std::mutex g_static_mu;
-void *g_static_ptr[kMaxDevices] = {};
-
-// Device address of g_static_scratch on the current device, looked up once per device.
+// Device address of g_static_scratch in the current device's context.  Looked up on every call
+// (a host-side table lookup once the module is loaded): a cached address would go stale when the
+// context is destroyed and re-created (cudaDeviceReset).
 int static_scratch_address(void **out) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) {
+    void *p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
+    if (e != cudaSuccess || !p) {
         g_last_cuda = (int)e;
         return TULA_ERR_CUDA;
     }
-    if (dev < 0 || dev >= kMaxDevices) return TULA_ERR_UNSUPPORTED;
-    std::lock_guard<std::mutex> lock(g_static_mu);
-    if (!g_static_ptr[dev]) {
-        void *p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_static_scratch);
-        if (e != cudaSuccess || !p) {
-            g_last_cuda = (int)e;
-            return TULA_ERR_CUDA;
-        }
-        g_static_ptr[dev] = p;
-    }
-    *out = g_static_ptr[dev];
+    *out = p;
+    return TULA_OK;
+}
+
+// The static array's error word (its layout's `err` section does not depend on the tensors).
+int static_scratch_error_word(unsigned **out) {
+    void *base = nullptr;
+    const int rc = static_scratch_address(&base);
+    if (rc) return rc;
+    *out = reinterpret_cast<unsigned *>(static_cast<char *>(base) + ws_layout(1, Plan{}).err);
     return TULA_OK;
 }
 
@@ -2112,22 +2137,58 @@ extern "C" int tula_ags_step_static_scratch(float *const *param_ptrs, float *con
                                             float weight_decay, const tula_ags_hparams *hp,
                                             void *stream) {
     Plan pl;
-    if (!hp || !valid_numels(numels, n_tensors, hp->K, &pl)) return TULA_ERR_ARG;
+    int rc = check_step_args(param_ptrs, grad_ptrs, mom_ptrs, numels, n_tensors, momentum, hp, &pl);
+    if (rc) return rc;
     const WsLayout L = ws_layout(n_tensors, pl);
     if (L.total > kStaticScratchBytes) return TULA_ERR_SCRATCH_LIMIT;
     void *scratch = nullptr;
-    int rc = static_scratch_address(&scratch);
+    rc = static_scratch_address(&scratch);
     if (rc) return rc;
-    // The array keeps the last call's contents: zero the counter, branch flag
-    // and error word (they precede the partial sums) before this call's kernels.
-    cudaError_t e = cudaMemsetAsync(scratch, 0, L.part1, static_cast<cudaStream_t>(stream));
+    // The array keeps the last call's contents: zero the tickets, the branch flag and the tile
+    // counters (they precede the partial sums) before this call's kernels.  The error word
+    // between them is left alone, so that a wait that ran out stays reported until
+    // tula_ags_static_scratch_error reads it.
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    char *b = static_cast<char *>(scratch);
+    cudaError_t e = cudaMemsetAsync(b, 0, L.err, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(b + L.tiles, 0, L.part1 - L.tiles, s);
     if (e != cudaSuccess) {
         g_last_cuda = (int)e;
         return TULA_ERR_CUDA;
     }
-    tula_ags_hparams local = *hp;
-    local.workspace = scratch;
-    local.workspace_bytes = kStaticScratchBytes;
-    return tula_ags_step(param_ptrs, grad_ptrs, mom_ptrs, numels, n_tensors, lr, momentum,
-                         weight_decay, &local, stream);
+    return run_step(param_ptrs, grad_ptrs, mom_ptrs, numels, n_tensors, lr, momentum,
+                    weight_decay, hp, scratch, pl, stream);
+}
+
+extern "C" int tula_ags_static_scratch_error(void *stream, int *error_out) {
+    if (!error_out) return TULA_ERR_ARG;
+    unsigned *word = nullptr;
+    int rc = static_scratch_error_word(&word);
+    if (rc) return rc;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    unsigned v = 0;
+    cudaError_t e = cudaMemcpyAsync(&v, word, sizeof(v), cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e == cudaSuccess && v) e = cudaMemsetAsync(word, 0, sizeof(v), s);
+    if (e == cudaSuccess && v) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) {
+        g_last_cuda = (int)e;
+        return TULA_ERR_CUDA;
+    }
+    *error_out = (int)v;
+    return TULA_OK;
+}
+
+extern "C" int tula_ags_static_scratch_check_wait_timeout(void *stream) {
+    unsigned *word = nullptr;
+    const int rc = static_scratch_error_word(&word);
+    if (rc) return rc;
+    k_wait_check<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(word);
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) {
+        g_last_cuda = (int)e;
+        return TULA_ERR_CUDA;
+    }
+    return TULA_OK;
 }

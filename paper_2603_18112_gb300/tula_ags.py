@@ -90,9 +90,12 @@ def lib() -> ctypes.CDLL:
     L.tula_ags_workspace_error.argtypes = [c_void_p, c_size_t, i64p, c_int, c_int,
                                            ctypes.POINTER(c_int)]
     L.tula_ags_check_wait_timeout.argtypes = [c_void_p, c_size_t, c_void_p]
+    L.tula_ags_static_scratch_error.argtypes = [c_void_p, ctypes.POINTER(c_int)]
+    L.tula_ags_static_scratch_check_wait_timeout.argtypes = [c_void_p]
     for name in ("tula_ags_workspace_size", "tula_ags_step", "tula_layer_stats",
                  "tula_ags_update_scale", "tula_ags_plan_chunks", "tula_ags_step_static_scratch",
-                 "tula_ags_workspace_error", "tula_ags_check_wait_timeout"):
+                 "tula_ags_workspace_error", "tula_ags_check_wait_timeout",
+                 "tula_ags_static_scratch_error", "tula_ags_static_scratch_check_wait_timeout"):
         getattr(L, name).restype = c_int
     _lib = L
     return L
@@ -141,6 +144,21 @@ def _stream_ptr(stream):
 def _check(rc, where):
     if rc != TULA_OK:
         raise TulaError(rc, where)
+
+
+def _replica_list(params, grads, hp, where, moms=None):
+    """grads[k][p] flattened k-major, after checking that it holds hp.K replicas of every
+    tensor (and one momentum buffer per tensor): the library reads K * n gradient pointers and
+    n momentum pointers, so a shorter list must not reach it."""
+    n = len(params)
+    if moms is not None and len(moms) != n:
+        raise ValueError(f"{where}: {len(moms)} momentum buffers for {n} tensors")
+    if hp is not None and hp.K != len(grads):
+        raise ValueError(f"{where}: hp.K = {hp.K} but {len(grads)} replica lists were given")
+    for k, r in enumerate(grads):
+        if len(r) != n:
+            raise ValueError(f"{where}: replica {k} has {len(r)} tensors, params has {n}")
+    return [grads[k][p] for k in range(len(grads)) for p in range(n)]
 
 
 # ---------------------------------------------------------------------------
@@ -216,8 +234,7 @@ def tula_ags_step(params, grads, moms, lr, momentum, weight_decay, hp: tula_ags_
     """One optimizer step.  params, moms: lists of n tensors (moms may be None);
     grads: K lists of n tensors (grads[k][p]); hp: tula_ags_hparams."""
     n = len(params)
-    K = len(grads)
-    flat = [grads[k][p] for k in range(K) for p in range(n)]
+    flat = _replica_list(params, grads, hp, "tula_ags_step", moms)
     rc = lib().tula_ags_step(_tensor_ptrs(params), _tensor_ptrs(flat),
                              _tensor_ptrs(moms) if moms is not None else None, _numels(params), n,
                              lr, momentum, weight_decay, ctypes.byref(hp), _stream_ptr(stream))
@@ -230,19 +247,34 @@ def tula_ags_step_static_scratch(params, grads, moms, lr, momentum, weight_decay
     the library's static device array (hp.workspace is ignored).  Calls on one device must not
     overlap on the GPU; make the first call on a device before any stream capture."""
     n = len(params)
-    K = len(grads)
-    flat = [grads[k][p] for k in range(K) for p in range(n)]
+    flat = _replica_list(params, grads, hp, "tula_ags_step_static_scratch", moms)
     rc = lib().tula_ags_step_static_scratch(
         _tensor_ptrs(params), _tensor_ptrs(flat), _tensor_ptrs(moms) if moms is not None else None,
         _numels(params), n, lr, momentum, weight_decay, ctypes.byref(hp), _stream_ptr(stream))
     _check(rc, "tula_ags_step_static_scratch")
 
 
+def tula_ags_static_scratch_error(stream=None) -> int:
+    """Reads and clears the static scratch's error word after the work on `stream`
+    (synchronous): 0 = every wait of the static-scratch steps since the last read completed."""
+    out = c_int(0)
+    _check(lib().tula_ags_static_scratch_error(_stream_ptr(stream), ctypes.byref(out)),
+           "tula_ags_static_scratch_error")
+    return out.value
+
+
+def tula_ags_static_scratch_check_wait_timeout(stream=None) -> None:
+    """The bounded-wait check against the static scratch's error word (about two seconds on
+    the GPU): afterwards tula_ags_static_scratch_error reports bit 0."""
+    _check(lib().tula_ags_static_scratch_check_wait_timeout(_stream_ptr(stream)),
+           "tula_ags_static_scratch_check_wait_timeout")
+
+
 def tula_layer_stats(params, grads, stats_out: torch.Tensor, workspace: torch.Tensor,
                      stream=None) -> None:
     n = len(params)
     K = len(grads)
-    flat = [grads[k][p] for k in range(K) for p in range(n)]
+    flat = _replica_list(params, grads, None, "tula_layer_stats")
     rc = lib().tula_layer_stats(_tensor_ptrs(params), _tensor_ptrs(flat), K, _numels(params), n,
                                 c_void_p(stats_out.data_ptr()), c_void_p(workspace.data_ptr()),
                                 workspace.numel() * workspace.element_size(), _stream_ptr(stream))
@@ -251,6 +283,9 @@ def tula_layer_stats(params, grads, stats_out: torch.Tensor, workspace: torch.Te
 
 def tula_ags_update_scale(g_small, g_large, hp: tula_ags_hparams, stream=None) -> None:
     n = len(g_small)
+    if len(g_large) != n:
+        raise ValueError(f"tula_ags_update_scale: {n} small-batch and {len(g_large)} "
+                         "large-batch tensors")
     rc = lib().tula_ags_update_scale(_tensor_ptrs(g_small), _tensor_ptrs(g_large),
                                      _numels(g_small), n, ctypes.byref(hp), _stream_ptr(stream))
     _check(rc, "tula_ags_update_scale")
@@ -276,6 +311,11 @@ class AGSOptimizerStep:
         self.moms = list(moms) if moms is not None else None
         self.n = len(self.params)
         self.K = len(self.grads)
+        if not 1 <= self.K <= TULA_MAX_K:
+            raise ValueError(f"AGSOptimizerStep: {self.K} replica lists (1 .. {TULA_MAX_K})")
+        if self.moms is not None and len(self.moms) != self.n:
+            raise ValueError(f"AGSOptimizerStep: {len(self.moms)} momentum buffers for "
+                             f"{self.n} tensors")
         dev = self.params[0].device
         self.hp = tula_ags_default_hparams(self.K)
         self.hp.rule = rule
@@ -303,7 +343,7 @@ class AGSOptimizerStep:
             self._scale_elem_tensors = list(scale_elem)
             self._scale_elem = _tensor_ptrs(self._scale_elem_tensors)
             self.hp.scale_elem = ctypes.cast(self._scale_elem, c_void_p).value
-        flat = [self.grads[k][p] for k in range(self.K) for p in range(self.n)]
+        flat = _replica_list(self.params, self.grads, self.hp, "AGSOptimizerStep")
         self._p = _tensor_ptrs(self.params)
         self._g = _tensor_ptrs(flat)
         self._m = _tensor_ptrs(self.moms) if self.moms is not None else None

@@ -146,3 +146,24 @@ def test_error_strings(lib):
     for code in (0, -1, -2, -3, -4, 99):
         assert isinstance(T.tula_ags_error_string(code), str)
     assert T.tula_ags_last_cuda_error() == 0
+
+
+def test_binding_refuses_replica_lists_that_do_not_match(lib):
+    """The wrappers check the list lengths before the C call: the library reads hp.K * n
+    gradient pointers and n momentum pointers, so a shorter list must never reach it."""
+    import torch
+    params = [torch.zeros(4), torch.zeros(4)]
+    grads = [[torch.zeros(4), torch.zeros(4)]]
+    hp = T.tula_ags_default_hparams(2)                       # K = 2, one replica list given
+    for fn in (T.tula_ags_step, T.tula_ags_step_static_scratch):
+        with pytest.raises(ValueError, match="replica"):
+            fn(params, grads, params, 0.1, 0.9, 0.0, hp)
+        hp1 = T.tula_ags_default_hparams(1)
+        with pytest.raises(ValueError, match="tensors"):     # replica 0 short of one tensor
+            fn(params, [[torch.zeros(4)]], params, 0.1, 0.9, 0.0, hp1)
+        with pytest.raises(ValueError, match="momentum"):
+            fn(params, grads, params[:1], 0.1, 0.9, 0.0, hp1)
+    with pytest.raises(ValueError):
+        T.AGSOptimizerStep(params, [[torch.zeros(4)]])
+    with pytest.raises(ValueError):
+        T.AGSOptimizerStep(params, [])

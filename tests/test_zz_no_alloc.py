@@ -40,6 +40,30 @@ def test_rejects_tensor_lists_beyond_the_static_scratch():
     assert "static scratch" in T.tula_ags_error_string(rc)
 
 
+def test_argument_errors_come_before_any_cuda_call():
+    """Host-only: every argument check of tula_ags_step runs before the static-scratch call
+    looks up its array or enqueues its memsets.  Without a GPU any CUDA call would fail with
+    TULA_ERR_CUDA, so TULA_ERR_ARG here shows that nothing reached CUDA."""
+    B.build()
+    lib = T.lib()
+    P = ctypes.c_void_p
+    ptrs = (P * 4)(*[0x100000 * (i + 1) for i in range(4)])
+    numels = (ctypes.c_int64 * 2)(5, 7)
+    hp = T.tula_ags_default_hparams(1)
+    hp.scale = 0x200000                                    # hp.state left NULL
+    rc = lib.tula_ags_step_static_scratch(ptrs, ptrs, ptrs, numels, 2, 0.1, 0.9, 0.0,
+                                          ctypes.byref(hp), None)
+    assert rc == T.TULA_ERR_ARG
+    hp.state, hp.rule = 0x300000, 9                        # bad enum
+    assert lib.tula_ags_step_static_scratch(ptrs, ptrs, ptrs, numels, 2, 0.1, 0.9, 0.0,
+                                            ctypes.byref(hp), None) == T.TULA_ERR_ARG
+    hp.rule = T.TULA_RULE_AGS
+    bad = (P * 4)(0x100000, 0x100002, 0x100000, 0x100000)  # misaligned second tensor
+    assert lib.tula_ags_step_static_scratch(bad, ptrs, ptrs, numels, 2, 0.1, 0.9, 0.0,
+                                            ctypes.byref(hp), None) == T.TULA_ERR_ARG
+    assert lib.tula_ags_static_scratch_error(None, None) == T.TULA_ERR_ARG
+
+
 def _model(wl, K, pset):
     buf = W.allocate(wl, "cuda", K=K, pset=pset)
     W.fill_state(buf, wl)
@@ -87,3 +111,51 @@ def test_static_scratch_step_matches_workspace_step():
         assert_norm_close(scale.cpu().numpy(), ref_step.scale.cpu().numpy(), where + " scale")
     assert state[3].item() == 1.0  # TULA_STATE_SCALED: the second call took the scaled branch
     assert np.isfinite(stats.cpu().numpy()).all()
+
+
+@pytest.mark.gpu
+def test_static_scratch_reports_a_wait_that_ran_out():
+    """Failure detection on the static scratch, without a fault: the bounded-wait check runs
+    out against the static array's error word (about two seconds), the word survives the next
+    static-scratch step (its memsets leave it alone), tula_ags_static_scratch_error reads bit 0
+    and clears it, and the step after that still matches tula_ags_step."""
+    B.build()
+    T.lib()
+    ps = W.param_set("resnet20")
+    ps.add((40000,), W.KIND_NORMAL)
+    wl = W.workload("resnet50", seed=78)
+    K = 2
+    ref = _model(wl, K, ps)
+    new = _model(wl, K, ps)
+    n = ps.n_tensors
+    ref_step = T.AGSOptimizerStep(ref.w, ref.g, ref.m, s_max=2.0)
+    hp = T.tula_ags_default_hparams(K)
+    scale = torch.ones(n, dtype=torch.float32, device="cuda")
+    state = torch.zeros(T.TULA_STATE_LEN, dtype=torch.float64, device="cuda")
+    hp.s_max = 2.0
+    hp.scale, hp.state = scale.data_ptr(), state.data_ptr()
+
+    def both_steps(seed_step):
+        for buf in (ref, new):
+            W.fill_grads(buf, wl, step=seed_step)
+        ref_step.step(wl.lr, wl.momentum, wl.weight_decay)
+        T.tula_ags_step_static_scratch(new.w, new.g, new.m, wl.lr, wl.momentum,
+                                       wl.weight_decay, hp)
+
+    torch.cuda.synchronize()
+    assert T.tula_ags_static_scratch_error() in (0, 1)  # whatever an earlier test left: cleared
+    assert T.tula_ags_static_scratch_error() == 0
+    both_steps(1)
+    assert T.tula_ags_static_scratch_error() == 0       # every wait of that step completed
+    T.tula_ags_static_scratch_check_wait_timeout()
+    both_steps(2)                                       # the word stays set through this step
+    assert T.tula_ags_static_scratch_error() == 1       # reported ...
+    assert T.tula_ags_static_scratch_error() == 0       # ... and cleared by the read
+    both_steps(3)
+    torch.cuda.synchronize()
+    assert T.tula_ags_static_scratch_error() == 0
+    assert torch.equal(new.g_flats[0], ref.g_flats[0]), "replica mean"
+    assert_f32_close(new.w_flat.cpu().numpy(), ref.w_flat.cpu().numpy(), "w")
+    assert_f32_close(new.m_flat.cpu().numpy(), ref.m_flat.cpu().numpy(), "m")
+    assert_state_close(state.cpu().numpy(), ref_step.state.cpu().numpy(), "state")
+    assert state[1].item() == 3.0
