@@ -35,14 +35,17 @@
  *     step may be partly applied: zero the workspace again before reusing it.
  *   - Element-wise arithmetic is IEEE fp32, one rounding per operation, in the
  *     order written below (no fused multiply-add).  Squared norms are fp32 sums
- *     within a tile (<= 2688 elements) added across tiles as float-float pairs
- *     (~48 significant bits), so their squares must lie in fp32's normal range
- *     (|x| within about 1e-19 .. 1e19).  Norms that feed a coefficient
- *     (gradscale refresh, LARS) split every square exactly into two fp32 parts,
- *     add them as float-float pairs per lane and in fp64 across lanes and tiles
- *     (relative error ~1e-14); a tile whose pairs cannot hold that (a square
- *     that overflows, or sums below 2^-77) is redone with exact fp64 squares,
- *     so these norms keep that precision over the whole fp32 range.
+ *     within a tile (<= 8192 elements; relative error below ~4e-6) added across
+ *     tiles in fp64.  A tile whose fp32 sums would overflow (a lane sum above
+ *     2^120) or lose precision to underflow (every lane sum below 2^-100, zero
+ *     included) is summed again with its elements scaled by an exact power of two,
+ *     and elements loaded one by one (tails, misaligned tensors) are squared in
+ *     fp64, so these norms hold over the whole fp32 range.  Norms that feed a
+ *     coefficient (gradscale refresh, LARS) split every square exactly into two
+ *     fp32 parts, add them as float-float pairs per lane and in fp64 across lanes
+ *     and tiles (relative error ~1e-14); a tile whose pairs cannot hold that (a
+ *     square that overflows, or sums below 2^-77) is redone with exact fp64
+ *     squares, so these norms keep that precision over the whole fp32 range.
  */
 #ifndef TULA_AGS_H
 #define TULA_AGS_H

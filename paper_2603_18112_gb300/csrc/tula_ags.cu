@@ -25,8 +25,9 @@
 // (cp.async.bulk ... mbarrier::complete_tx), one copy per stream issued by one
 // lane each; consumer warps, each owning whole stages, compute from shared
 // memory and release the stage through an mbarrier.  Tile partials are fp32
-// sums within a tile, carried as float-float pairs (fp64 in the precise mode
-// for norms that feed a coefficient); only plain stores leave a tile.
+// sums within a tile (float-float pairs per lane in the precise mode for norms
+// that feed a coefficient), range-checked per tile and stored as fp64; only
+// plain stores leave a tile.
 //
 // Every mbarrier wait is bounded; a wait that runs out sets an error word in
 // the workspace (tula_ags_workspace_error) and the CTA drains its copies in
@@ -148,10 +149,10 @@ struct Scalars {
     unsigned *err;   // [0]: bounded waits that ran out (sticky until read)
     unsigned *sctr1; // [tensor]: segments combined, pass 1
     unsigned *sctr2; // [tensor]: segments combined, pass 2
-    float2 *part1;   // [tile][kAcc], pass 1 (float-float sums)
-    float2 *part2;   // [tile], pass 2 (|w|^2)
-    float2 *spart1;  // [segment][kAcc], pass 1
-    float2 *spart2;  // [segment], pass 2
+    double *part1;   // [tile][kAcc], pass 1
+    double *part2;   // [tile], pass 2 (|w|^2)
+    double *spart1;  // [segment][kAcc], pass 1
+    double *spart2;  // [segment], pass 2
     double *tsum;    // [tensor][kTsum]: |gbar|^2, |g_0|^2, |w|^2
     float *cand;     // [tensor]: c_p of the scaled branch (AGS: the old gradscale)
     unsigned *tiles; // [2 * pass]: next tile to claim, [2 * pass + 1]: CTAs finished
@@ -169,11 +170,6 @@ __device__ __forceinline__ void st_keep(float *p, float4 v) {
 }
 // 8-byte store that asks L2 to keep the line: tile partials, read back by the
 // combine kernel right after the streaming kernel that writes them.
-__device__ __forceinline__ void st_keep_l2(float2 *p, float2 v, uint64_t policy) {
-    asm volatile("st.global.L2::cache_hint.v2.f32 [%0], {%1, %2}, %3;" ::"l"(p), "f"(v.x), "f"(v.y),
-                 "l"(policy)
-                 : "memory");
-}
 __device__ __forceinline__ void st_keep_l2(double *p, double v, uint64_t policy) {
     asm volatile("st.global.L2::cache_hint.f64 [%0], %1, %2;" ::"l"(p), "d"(v), "l"(policy) : "memory");
 }
@@ -249,8 +245,40 @@ __device__ __forceinline__ void warp_sums(float (&v)[R]) {
     }
 }
 
+// Warp reduce-scatter of R values per lane (R a power of two, <= 32): each of log2(R) halving
+// steps sends half of a lane's values to the lane `off` away and keeps the sums of the other
+// half; the remaining steps add the one value left across the lanes still sharing it.
+// Afterwards every lane holds the warp total of value `index` (bits of the lane id reversed):
+// with R = 16, lanes 2i and 2i + 1 hold the same one.  16 + 1 shuffles for R = 16 instead of
+// the 5 R of a tree per value, so the owners of R sums can store them at once.  The order of
+// the additions is fixed (results do not depend on timing), and the two lanes that end with
+// the same sum add the same two terms.
+__device__ __forceinline__ float add_rn(float a, float b) { return __fadd_rn(a, b); }
+__device__ __forceinline__ double add_rn(double a, double b) { return __dadd_rn(a, b); }
+template <int R, typename T>
+__device__ __forceinline__ T warp_reduce_scatter(T (&v)[R], int &index) {
+    static_assert(R >= 1 && R <= 32 && (R & (R - 1)) == 0, "R: a power of two <= 32");
+    const int lane = threadIdx.x & 31;
+    int idx = 0, off = 16;
+#pragma unroll
+    for (int h = R / 2; h >= 1; h >>= 1, off >>= 1) {
+        const bool up = (lane & off) != 0;
+#pragma unroll
+        for (int j = 0; j < h; ++j) {
+            const T send = up ? v[j] : v[j + h];
+            const T keep = up ? v[j + h] : v[j];
+            v[j] = add_rn(keep, __shfl_xor_sync(kFull, send, off));
+        }
+        if (up) idx += h;
+    }
+#pragma unroll
+    for (; off >= 1; off >>= 1) v[0] = add_rn(v[0], __shfl_xor_sync(kFull, v[0], off));
+    index = idx;
+    return v[0];
+}
+
 // Float-float numbers (hi, lo as a float2, value hi + lo, |lo| <= ulp(hi) / 2)
-// carry the partial sums between kernels: they hold ~48 significant bits and
+// carry the precise path's per-lane sums: they hold ~48 significant bits and
 // add on the FP32 pipes, where an fp64 add costs ~64x more on this part.
 // Knuth's TwoSum: s + e == a + b exactly.
 __device__ __forceinline__ float2 two_sum(float a, float b) {
@@ -313,43 +341,54 @@ __device__ __forceinline__ bool dw_lane_ok(float2 v) {
     return v.x >= 0x1p-77f && v.x <= 3.0e38f;  // false for 0, tiny sums, inf and NaN
 }
 
-// Partial sums travel as float-float pairs, or as fp64 where the norms feed a
-// coefficient (precise mode): Part<P>::T is the stored type, zero/add/tree work
-// on it.  Both are 8 bytes, so the workspace layout is the same.
-template <bool P>
-struct Part;
-template <>
-struct Part<false> {
-    using T = float2;
-    static __device__ __forceinline__ T zero() { return make_float2(0.f, 0.f); }
-    static __device__ __forceinline__ T add(T a, T b) { return ff_add(a, b); }
-    static __device__ __forceinline__ double value(T a) { return ff_to_double(a); }
-};
-template <>
-struct Part<true> {
-    using T = double;
-    static __device__ __forceinline__ T zero() { return 0.0; }
-    static __device__ __forceinline__ T add(T a, T b) { return __dadd_rn(a, b); }
-    static __device__ __forceinline__ double value(T a) { return a; }
-};
-// Fixed-tree warp sum of R float-float values (lane 0 gets the sums).
-template <int R>
-__device__ __forceinline__ void warp_sums_ff(double (&v)[R]) {
-    warp_sums<R>(v);
+// Exact powers of two (k within the normal range of the type).
+__device__ __forceinline__ float pow2f(int k) { return __int_as_float((k + 127) << 23); }
+__device__ __forceinline__ double pow2d(int k) {
+    return __longlong_as_double((long long)(k + 1023) << 52);
 }
-template <int R>
-__device__ __forceinline__ void warp_sums_ff(float2 (&v)[R]) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        float2 t[R];
-#pragma unroll
-        for (int r = 0; r < R; ++r) {
-            t[r].x = __shfl_down_sync(kFull, v[r].x, o);
-            t[r].y = __shfl_down_sync(kFull, v[r].y, o);
-        }
-#pragma unroll
-        for (int r = 0; r < R; ++r) v[r] = ff_add(v[r], t[r]);
-    }
+
+// Range of a tile's fp32 sums of squares, decided for the whole warp from the largest lane
+// sum v (>= 0, or NaN): 0 when every lane sum is safe as it stands, else the exponent e of a
+// power-of-two scaling 2^e to apply to the elements before squaring them again.
+//  * max in [2^-100, 2^120]: nothing overflows (32 lanes add to < 2^125), and squares or partial
+//    sums that fell below fp32's normal range err by at most 2^-150 each, < 2^-38 of the tile
+//    sum: kept.
+//  * max above 2^120, inf or NaN: a square or a sum reached fp32's top.  Scaled by 2^-72 every
+//    finite element is below 2^56, its square below 2^112, a lane's sum of up to 256 squares
+//    below 2^120; what the scaling pushes below 2^-149 has a square under 2^-254 of the tile
+//    sum.  Inf and NaN stay inf and NaN.
+//  * max below 2^-100 (zero included): every element is below 2^-50 in magnitude (a sum of
+//    squares is at least its largest term), so 2^100 x is exact, below 2^50, and its square is a
+//    normal number unless x is 0.
+constexpr int kScaleUp = 100, kScaleDown = -72;
+// Two-bit codes of those exponents, for the partial sums a batch of tiles carries.
+__device__ __forceinline__ unsigned scale_code(int e) { return e == 0 ? 0u : (e > 0 ? 1u : 2u); }
+__device__ __forceinline__ int scale_exp(unsigned code) {
+    return code == 0u ? 0 : (code == 1u ? kScaleUp : kScaleDown);
+}
+__device__ __forceinline__ bool sq_in_range(float v) {
+    return v >= 0x1p-100f && v <= 0x1p120f;  // false for NaN
+}
+__device__ __forceinline__ int sq_range_exp(float v) {
+    const unsigned m = __reduce_max_sync(kFull, __float_as_uint(v));
+    if (m > __float_as_uint(0x1p120f)) return kScaleDown;
+    if (m < __float_as_uint(0x1p-100f)) return kScaleUp;
+    return 0;
+}
+// x * 2^k as a double, exactly, built on the integer pipes (GB300's FP64 pipe is slow): x is a
+// tile's range-checked fp32 sum, i.e. zero, normal, inf or NaN; a subnormal x (which the range
+// check rules out) takes the fp64 route.
+__device__ __forceinline__ double widen_scaled(float x, int k) {
+    const unsigned u = __float_as_uint(x);
+    const unsigned e = (u >> 23) & 0xffu;
+    const unsigned long long sign = (unsigned long long)(u >> 31) << 63;
+    const unsigned long long man = (unsigned long long)(u & 0x7fffffu) << 29;
+    if (e == 0u) return man ? __dmul_rn((double)x, pow2d(k)) : __longlong_as_double((long long)sign);
+    const unsigned long long ex = e == 0xffu ? 0x7ffull : (unsigned long long)((int)e - 127 + 1023 + k);
+    return __longlong_as_double((long long)(sign | (ex << 52) | man));
+}
+__device__ __forceinline__ float4 mul4(float4 v, float f) {
+    return make_float4(__fmul_rn(v.x, f), __fmul_rn(v.y, f), __fmul_rn(v.z, f), __fmul_rn(v.w, f));
 }
 
 // ----------------------------------------------------------------------------
@@ -709,7 +748,10 @@ __device__ __forceinline__ int next_tile(const Scalars &sc, int j, uint64_t *ful
 // group sums, then a 5-level tree across lanes, a relative error below 71 ulp
 // (4e-6) of the tile's sum; tiles are combined in fp64.  That is what the
 // variability metric and the statistics need, and it keeps GB300's slow FP64
-// pipe out of the streaming loop.
+// pipe out of the streaming loop.  One warp vote per tile (sq_range_exp) keeps
+// it valid over the whole fp32 range: a tile whose fp32 sums would overflow or
+// lose precision to underflow is summed again from shared memory with its
+// elements scaled by an exact power of two, and the scaling is undone in fp64.
 // Pointer roles per tensor: [0, K) replicas, KS = w, KS + 1 = g_small.
 // Stage streams: replicas 0..K-1, then w (RW), then g_small (SS).
 
@@ -777,11 +819,43 @@ __device__ __noinline__ D3 tile_cols_fp64(uint32_t stage, int chunk, int nv, con
     return r;
 }
 
-// Per-lane partial sums of one tile (not yet reduced across the warp).
+// A tile's shared-memory columns again in fp32, every element multiplied by an exact power of
+// two first (sq_range_exp): the default path's fallback when a tile's fp32 sums of squares
+// would overflow or lose their precision to underflow.  Returns this lane's sums of the scaled
+// squares.  Out of line, so that the streaming loop keeps its shape.
+struct F3 {
+    float g, s, w;
+};
+template <int KT, bool RW, bool SS>
+__device__ __noinline__ F3 tile_cols_scaled(uint32_t stage, int chunk, int nv, const Scalars &sc,
+                                            float fg, float fs, float fw) {
+    const int lane = threadIdx.x & 31;
+    const int K = KT > 0 ? KT : sc.K;
+    const uint32_t sw_s = stage + (uint32_t)(K * chunk * 4);
+    const uint32_t ss_s = stage + (uint32_t)((K + (RW ? 1 : 0)) * chunk * 4);
+    F3 r = {0.f, 0.f, 0.f};
+    for (int v = lane; v < nv; v += 32) {
+        const float4 x0 = lds4(stage + (uint32_t)(16 * v));
+        float4 s = x0;
+        for (int k = 1; k < K; ++k) s = add4(s, lds4(stage + (uint32_t)((k * chunk + 4 * v) * 4)));
+        if (K > 1) s = mean4<KT>(s, sc);
+        r.g = sq4(r.g, mul4(s, fg));
+        if (K > 1) r.s = sq4(r.s, mul4(x0, fs));
+        if (SS) r.s = sq4(r.s, mul4(lds4(ss_s + (uint32_t)(16 * v)), fs));
+        if (RW) r.w = sq4(r.w, mul4(lds4(sw_s + (uint32_t)(16 * v)), fw));
+    }
+    return r;
+}
+
+// Per-lane partial sums of one tile (not yet reduced across the warp).  Precise mode (PR):
+// accd holds the lane's fp64 sums.  Default mode: accf holds the lane's fp32 sums over the
+// tile's shared-memory columns, scaled by 2^(2 acce) (acce is the same in every lane), and accd
+// the lane's exact fp64 sums over the elements loaded directly (tail, misaligned tensor).
 template <int KT, bool WM, bool RW, bool SS, bool PR>
 __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const float *const *ptr,
                                             const TilePos &q, int nv, const Scalars &sc,
-                                            double (&accd)[kAcc], float (&accf)[kAcc]) {
+                                            double (&accd)[kAcc], float (&accf)[kAcc],
+                                            int (&acce)[kAcc], unsigned &ecode, bool &tail) {
     constexpr int KS = P1<KT>::KS;
     const int lane = threadIdx.x & 31;
     const int K = KT > 0 ? KT : sc.K;
@@ -792,8 +866,10 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
     dw_zero(ag);
     dw_zero(as);
     dw_zero(aw);
-    double rg = 0.0, rs = 0.0, rw = 0.0;  // precise (PR) sums of the elements loaded directly
+    double rg = 0.0, rs = 0.0, rw = 0.0;  // exact fp64 sums of the elements loaded directly
     const int ncols = nv;                 // the shared-memory columns (nv is reused below)
+    tail = false;                         // the tile has elements loaded one by one
+    ecode = 0u;                           // scale_code of acce[a] in bits 2a, 2a + 1
     float fg = 0.f, fs = 0.f, fw = 0.f;   // fp32 sums (not PR)
 
     if constexpr (KT > 0) {
@@ -856,7 +932,9 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
                 if (RW) fw = __fadd_rn(fw, pw);
             }
         }
-        // Tail (< 4 elements) or a misaligned tensor: plain loads from global memory.
+        // Tail (< 4 elements) or a misaligned tensor: plain loads from global memory, exact
+        // squares in fp64 (this is where replica 0 is overwritten, so there is no second look).
+        tail = q.begin + 4 * (long long)nv < q.end;  // the same in every lane
         for (long long j = q.begin + 4 * (long long)nv + lane; j < q.end; j += 32) {
             const float x0 = __ldcs(ptr[0] + j);
             float s = x0;
@@ -867,17 +945,10 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
             }
             const float y_s = SS ? __ldcs(ptr[KS + 1] + j) : 0.f;
             const float y_w = RW ? __ldcs(ptr[KS] + j) : 0.f;
-            if (PR) {
-                if (K > 1) rs = __fma_rn((double)x0, (double)x0, rs);
-                rg = __fma_rn((double)s, (double)s, rg);
-                if (SS) rs = __fma_rn((double)y_s, (double)y_s, rs);
-                if (RW) rw = __fma_rn((double)y_w, (double)y_w, rw);
-            } else {
-                if (K > 1) fs = __fmaf_rn(x0, x0, fs);
-                fg = __fmaf_rn(s, s, fg);
-                if (SS) fs = __fmaf_rn(y_s, y_s, fs);
-                if (RW) fw = __fmaf_rn(y_w, y_w, fw);
-            }
+            if (K > 1) rs = __fma_rn((double)x0, (double)x0, rs);
+            rg = __fma_rn((double)s, (double)s, rg);
+            if (SS) rs = __fma_rn((double)y_s, (double)y_s, rs);
+            if (RW) rw = __fma_rn((double)y_w, (double)y_w, rw);
         }
     }
     if (PR) {
@@ -900,9 +971,60 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
         accd[1] = (K > 1 || SS) ? __dadd_rn(cs, rs) : accd[0];  // K = 1: replica 0 is the mean
         accd[2] = RW ? __dadd_rn(cw, rw) : 0.0;
     } else {
+        // The warp is converged again here; ncols is the same in every lane.
+        int eg = 0, es = 0, ew = 0;
+        // One vote per tile; the warp maxima only when some lane is out of range.  A lane
+        // without columns (lane >= ncols) has nothing to check.
+        const bool lane_ok = lane >= ncols || (sq_in_range(fg) && (!(K > 1 || SS) || sq_in_range(fs)) &&
+                                               (!RW || sq_in_range(fw)));
+        if (ncols > 0 && !__all_sync(kFull, lane_ok)) {
+            eg = sq_range_exp(fg);
+            if (K > 1 || SS) es = sq_range_exp(fs);
+            if (RW) ew = sq_range_exp(fw);
+            if (eg | es | ew) {
+                const F3 r = tile_cols_scaled<KT, RW, SS>(stage, chunk, ncols, sc, pow2f(eg),
+                                                          pow2f(es), pow2f(ew));
+                if (eg) fg = r.g;
+                if (es) fs = r.s;
+                if (ew) fw = r.w;
+                const bool own = K > 1 || SS;
+                ecode = scale_code(eg) | scale_code(own ? es : eg) << 2 | scale_code(ew) << 4;
+            }
+        }
+        const bool own_s = K > 1 || SS;  // K = 1: replica 0 is the mean
         accf[0] = fg;
-        accf[1] = (K > 1 || SS) ? fs : fg;
+        acce[0] = eg;
+        accd[0] = rg;
+        accf[1] = own_s ? fs : fg;
+        acce[1] = own_s ? es : eg;
+        accd[1] = own_s ? rs : rg;
         accf[2] = fw;
+        acce[2] = ew;
+        accd[2] = rw;
+    }
+}
+
+static_assert(kPend == 4, "the owner lanes below pick one of four tiles");
+
+// A default-mode tile with elements loaded one by one (the last tile of a tensor whose size is
+// not a multiple of 4, or a misaligned tensor): its sums are reduced across the warp at once,
+// fp32 part and fp64 part, and lane 0 stores the tile's kAcc partials.
+__device__ __noinline__ void store_tile_now(double *P, const float (&accf)[kAcc],
+                                            const int (&acce)[kAcc], const double (&accd)[kAcc],
+                                            uint64_t keep) {
+    float f[kAcc];
+    double d[kAcc];
+#pragma unroll
+    for (int a = 0; a < kAcc; ++a) {
+        f[a] = accf[a];
+        d[a] = accd[a];
+    }
+    warp_sums<kAcc>(f);
+    warp_sums<kAcc>(d);
+    if ((threadIdx.x & 31) == 0) {
+#pragma unroll
+        for (int a = 0; a < kAcc; ++a)
+            st_keep_l2(P + a, __dadd_rn(widen_scaled(f[a], -2 * acce[a]), d[a]), keep);
     }
 }
 
@@ -949,19 +1071,28 @@ __global__ void __launch_bounds__(Ring1For<PR>::kThreads, 1)
     const int cw = warp - 1;
     TensorCache tc;
     bool stop = false;
+    const uint64_t keep = policy_evict_last();
+    // The partial sums of a batch of kPend tiles are reduced across the warp together
+    // (reduce-scatter, kRS values with padding) and stored by the lanes that own them.
+    constexpr int kRS = 16;
+    static_assert(kPend * kAcc <= kRS, "one reduce-scatter per batch");
     for (int jb = cw; !stop; jb += R1::kConsumers * kPend) {
-        double pendd[PR ? kPend * kAcc : 1];
-        float pendf[PR ? 1 : kPend * kAcc];
+        // PR: the lanes' fp64 sums.  Default: fp32 sums of the shared-memory columns, scaled by
+        // 2^(2e) with e coded in two bits per value in `ecode` (same in every lane); a tile with
+        // elements loaded one by one (fp64, rare) is stored at once instead (store_tile_now).
+        double pendd[PR ? kRS : 1];
+        float pendf[PR ? 1 : kRS];
+        unsigned ecode = 0u;
         int ptile[kPend];
+#pragma unroll
+        for (int i = 0; i < kRS; ++i) {
+            if constexpr (PR) pendd[i] = 0.0;
+            else pendf[i] = 0.f;
+        }
 #pragma unroll
         for (int p = 0; p < kPend; ++p) {
             const int j = jb + p * R1::kConsumers;
             ptile[p] = -1;
-#pragma unroll
-            for (int a = 0; a < kAcc; ++a) {
-                if constexpr (PR) pendd[p * kAcc + a] = 0.0;
-                else pendf[p * kAcc + a] = 0.f;
-            }
             if (stop) continue;
             // A round-robin tile is located before its wait, a claimed one after.
             int c = j < js ? static_tile(j) : -1;
@@ -980,31 +1111,39 @@ __global__ void __launch_bounds__(Ring1For<PR>::kThreads, 1)
             const float *const *ptr = tab.ptr[q.t];
             double accd[kAcc];
             float accf[kAcc];
+            int acce[kAcc];
+            unsigned tcode;
+            bool tile_tail;
             reduce_tile<KT, WM, RW, SS, PR>(ring + (uint32_t)s * R1::kStageBytes, chunk, ptr, q,
-                                            tc.nv, sc, accd, accf);
+                                            tc.nv, sc, accd, accf, acce, tcode, tile_tail);
             __syncwarp();
             if (lane == 0) mbar_arrive(&empty[s]);
-            ptile[p] = tab.c0 + c;
+            if constexpr (PR) {
+                ptile[p] = tab.c0 + c;
 #pragma unroll
-            for (int a = 0; a < kAcc; ++a) {
-                if constexpr (PR) pendd[p * kAcc + a] = accd[a];
-                else pendf[p * kAcc + a] = accf[a];
+                for (int a = 0; a < kAcc; ++a) pendd[p * kAcc + a] = accd[a];
+            } else if (tile_tail) {
+                store_tile_now(sc.part1 + (size_t)(tab.c0 + c) * kAcc, accf, acce, accd, keep);
+            } else {
+                ptile[p] = tab.c0 + c;
+#pragma unroll
+                for (int a = 0; a < kAcc; ++a) pendf[p * kAcc + a] = accf[a];
+                ecode |= tcode << (2 * kAcc * p);
             }
         }
-        if constexpr (PR) warp_sums<kPend * kAcc>(pendd);
-        else warp_sums<kPend * kAcc>(pendf);
-        if (lane == 0) {
-#pragma unroll
-            for (int p = 0; p < kPend; ++p)
-                if (ptile[p] >= 0) {
-                    float2 *P = sc.part1 + (size_t)ptile[p] * kAcc;
-                    const uint64_t keep = policy_evict_last();
-#pragma unroll
-                    for (int a = 0; a < kAcc; ++a) {
-                        if constexpr (PR) st_keep_l2(reinterpret_cast<double *>(P) + a, pendd[p * kAcc + a], keep);
-                        else st_keep_l2(P + a, make_float2(pendf[p * kAcc + a], 0.f), keep);
-                    }
-                }
+        int idx;
+        double v;
+        if constexpr (PR) {
+            v = warp_reduce_scatter<kRS>(pendd, idx);
+        } else {
+            const float f = warp_reduce_scatter<kRS>(pendf, idx);
+            v = widen_scaled(f, -2 * scale_exp((ecode >> (2 * idx)) & 3u));
+        }
+        // lanes 2i hold value i = p * kAcc + a of the batch
+        if ((lane & 1) == 0 && idx < kPend * kAcc) {
+            const int p = idx / kAcc, a = idx - p * kAcc;
+            const int t = p == 0 ? ptile[0] : p == 1 ? ptile[1] : p == 2 ? ptile[2] : ptile[3];
+            if (t >= 0) st_keep_l2(sc.part1 + (size_t)t * kAcc + a, v, keep);
         }
         if (stop) break;
     }
@@ -1088,28 +1227,30 @@ __device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, dou
     }
 }
 
+// Eight values added in a fixed pairwise tree (three dependent adds instead of eight).
+__device__ __forceinline__ double sum8(const double (&x)[8]) {
+    return __dadd_rn(__dadd_rn(__dadd_rn(x[0], x[1]), __dadd_rn(x[2], x[3])),
+                     __dadd_rn(__dadd_rn(x[4], x[5]), __dadd_rn(x[6], x[7])));
+}
+
 // |G|^2, Delta (Eq. 5) and the branch of Algorithm 1 (one warp, after every
 // segment's |gbar|^2 is in sc.spart1; segments in index order, then a fixed tree).
-template <bool PREC>
 __device__ void finalize_step(const Scalars &sc, double g2_prev, double steps) {
-    using PT = Part<PREC>;
-    using T = typename PT::T;
-    const T *spart = reinterpret_cast<const T *>(sc.spart1);
+    const double *spart = sc.spart1;
     const int lane = threadIdx.x & 31;
-    T v[1] = {PT::zero()};
+    double v[1] = {0.0};
     for (int g0 = 0; g0 < sc.n_seg1; g0 += 8 * 32) {  // 8 loads in flight per lane
-        T x[8];
+        double x[8];
 #pragma unroll
         for (int u = 0; u < 8; ++u) {
             const int g = g0 + lane + 32 * u;
-            x[u] = g < sc.n_seg1 ? __ldcg(&spart[(size_t)g * kAcc + 0]) : PT::zero();
+            x[u] = g < sc.n_seg1 ? __ldcg(&spart[(size_t)g * kAcc + 0]) : 0.0;
         }
-#pragma unroll
-        for (int u = 0; u < 8; ++u) v[0] = PT::add(v[0], x[u]);
+        v[0] = __dadd_rn(v[0], sum8(x));
     }
-    warp_sums_ff<1>(v);
+    warp_sums<1>(v);
     if (lane != 0) return;
-    const double g2 = PT::value(v[0]);
+    const double g2 = v[0];
     // no previous step -> +inf (sensitive)
     const double dv = steps == 0.0 ? (double)INFINITY : fabs((g2 - g2_prev) / g2_prev);
     int scaled;
@@ -1124,11 +1265,9 @@ __device__ void finalize_step(const Scalars &sc, double g2_prev, double steps) {
     sc.done[1] = 0u;  // re-arm for the next call
 }
 
-template <int NA, bool PREC>
+template <int NA>
 __global__ void __launch_bounds__(32 * kCombWarps)
     k_combine(const __grid_constant__ CombTable tab, const __grid_constant__ Scalars sc) {
-    using PT = Part<PREC>;
-    using T = typename PT::T;
     // Everything that does not come from the kernel before is read ahead of the
     // wait for it (this kernel is launched early and waits through most of the
     // previous one): the segment's place in the table and, in a step, the old
@@ -1153,32 +1292,30 @@ __global__ void __launch_bounds__(32 * kCombWarps)
     // overwrites the tile partials this kernel reads).
     if (sc.mode == kModeStep || NA == 1) grid_launch_dependents();
     if (!active) return;
-    const T *part = reinterpret_cast<const T *>(NA == kAcc ? sc.part1 : sc.part2);
-    T *spart = reinterpret_cast<T *>(NA == kAcc ? sc.spart1 : sc.spart2);
+    const double *part = NA == kAcc ? sc.part1 : sc.part2;
+    double *spart = NA == kAcc ? sc.spart1 : sc.spart2;
     unsigned *sctr = NA == kAcc ? sc.sctr1 : sc.sctr2;
 
     // The segment's tiles: lane i adds tiles i, i + 32, ... in order (8 loads in
     // flight), then a fixed tree across the warp.
-    T v[NA];
+    double v[NA];
 #pragma unroll
-    for (int a = 0; a < NA; ++a) v[a] = PT::zero();
+    for (int a = 0; a < NA; ++a) v[a] = 0.0;
     int i = lane;
     for (; i + 7 * 32 < n; i += 8 * 32) {
-        T x[8][NA];
+        double x[NA][8];
 #pragma unroll
         for (int u = 0; u < 8; ++u)
 #pragma unroll
-            for (int a = 0; a < NA; ++a) x[u][a] = part[(first + i + 32 * u) * NA + a];
+            for (int a = 0; a < NA; ++a) x[a][u] = part[(first + i + 32 * u) * NA + a];
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
-#pragma unroll
-            for (int a = 0; a < NA; ++a) v[a] = PT::add(v[a], x[u][a]);
+        for (int a = 0; a < NA; ++a) v[a] = __dadd_rn(v[a], sum8(x[a]));
     }
     for (; i < n; i += 32) {
 #pragma unroll
-        for (int a = 0; a < NA; ++a) v[a] = PT::add(v[a], part[(first + i) * NA + a]);
+        for (int a = 0; a < NA; ++a) v[a] = __dadd_rn(v[a], part[(first + i) * NA + a]);
     }
-    warp_sums_ff<NA>(v);
+    warp_sums<NA>(v);
 
     // The branch needs only |G|^2, so it does not wait for the tensors: in a step,
     // every segment posts its sums and takes a ticket over all segments, and the
@@ -1201,27 +1338,27 @@ __global__ void __launch_bounds__(32 * kCombWarps)
     }
     if (last_all) {
         fence_acq_rel();
-        finalize_step<PREC>(sc, g2_prev, steps);
+        finalize_step(sc, g2_prev, steps);
     }
     if (!last_seg) return;
     if (nseg > 1) {
         fence_acq_rel();
 #pragma unroll
-        for (int a = 0; a < NA; ++a) v[a] = PT::zero();
+        for (int a = 0; a < NA; ++a) v[a] = 0.0;
         for (int j = lane; j < nseg; j += 32) {
 #pragma unroll
-            for (int a = 0; a < NA; ++a) v[a] = PT::add(v[a], __ldcg(&spart[(sg0 + j) * NA + a]));
+            for (int a = 0; a < NA; ++a) v[a] = __dadd_rn(v[a], __ldcg(&spart[(sg0 + j) * NA + a]));
         }
-        warp_sums_ff<NA>(v);
+        warp_sums<NA>(v);
         if (lane == 0) sctr[tg] = 0u;  // re-arm
     }
 
     // This warp holds tensor tg's sums (lane 0).
     if constexpr (NA == kAcc) {
-        tensor_done(sc, tg, PT::value(v[0]), PT::value(v[1]), PT::value(v[2]), scale_old);
+        tensor_done(sc, tg, v[0], v[1], v[2], scale_old);
     } else {
         // lanes 0 and 1 take the two square roots in one instruction
-        const double sw = __shfl_sync(kFull, PT::value(v[0]), 0);
+        const double sw = __shfl_sync(kFull, v[0], 0);
         const double sg = sc.tsum[(size_t)tg * kTsum + 0];
         const double r = sqrt(lane == 0 ? sw : sg);
         const double nw = __shfl_sync(kFull, r, 0), ng = __shfl_sync(kFull, r, 1);
@@ -1266,6 +1403,26 @@ __device__ __forceinline__ float update4(float4 g4, float4 w4, float4 m4, float4
     st_stream(wp, w4);
     if (HM) st_stream(mp, m4);
     return pw;
+}
+
+// |w|^2 of a tile's shared-memory w columns in fp32, every element multiplied by the power of
+// two f first (sq_range_exp): the statistics' fallback when the tile's fp32 sums would overflow
+// or lose their precision to underflow.  Out of line, like tile_cols_scaled.
+__device__ __noinline__ float w_cols_scaled(uint32_t w_stage, int nv, float f) {
+    float a = 0.f;
+    for (int v = threadIdx.x & 31; v < nv; v += 32) a = sq4(a, mul4(lds4(w_stage + (uint32_t)(16 * v)), f));
+    return a;
+}
+
+// A tile of the update with elements loaded one by one: its |w|^2 (fp32 part scaled by 2^(2e),
+// fp64 part) reduced across the warp at once and stored by lane 0.
+__device__ __noinline__ void store_w_tile_now(double *P, float aw, int e, double awt) {
+    float f[1] = {aw};
+    double d[1] = {awt};
+    warp_sums<1>(f);
+    warp_sums<1>(d);
+    if ((threadIdx.x & 31) == 0)
+        st_keep_l2(P, __dadd_rn(widen_scaled(f[0], -2 * e), d[0]), policy_evict_last());
 }
 
 template <bool HM, bool PE, bool SW>
@@ -1320,7 +1477,10 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
     float cand = 0.f;
     bool stop = false;
     for (int jb = cw; !stop; jb += Ring2::kConsumers * kPend) {
+        // fp32 |w|^2 of the tiles' shared-memory columns, scaled by 2^(2e) (e coded in `ecode`);
+        // a tile with elements loaded one by one (fp64, rare) is stored at once instead.
         float pend[kPend];
+        unsigned ecode = 0u;
         int ptile[kPend];
 #pragma unroll
         for (int p = 0; p < kPend; ++p) {
@@ -1355,7 +1515,8 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
             float *wp = const_cast<float *>(ptr[1]) + q.begin;
             float *mp = HM ? const_cast<float *>(ptr[2]) + q.begin : nullptr;
             const float4 cdef = PE ? make_float4(1.f, 1.f, 1.f, 1.f) : make_float4(ct, ct, ct, ct);
-            float aw = 0.f;  // fp32 |w|^2 of the tile (statistics only)
+            float aw = 0.f;    // fp32 |w|^2 of the tile's columns (statistics only)
+            double awt = 0.0;  // exact fp64 |w|^2 of its tail
             if (nv == CH / 4) {
                 // Two columns per step of a rolled loop (unrolled over the tile, the body
                 // outgrew the instruction cache: 82.5 -> 75.5 us per ResNet-50 update pass).
@@ -1391,30 +1552,47 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
                     if (SW) aw = __fadd_rn(aw, pw);
                 }
             }
+            // The warp is converged again; nv is the same in every lane.  The stage still holds
+            // the tile's w before the update.
+            int ew = 0;
+            if (SW && nv > 0 && !__all_sync(kFull, lane >= nv || sq_in_range(aw))) {
+                ew = sq_range_exp(aw);
+                if (ew) aw = w_cols_scaled(stage + w_off, nv, pow2f(ew));
+            }
             __syncwarp();
             if (lane == 0) mbar_arrive(&empty[s]);
             const long long n = q.end - q.begin;
+            const bool tile_tail = 4 * (long long)nv < n;  // the same in every lane
             for (long long jj = 4 * (long long)nv + lane; jj < n; jj += 32) {
                 const float g = __ldcs(ptr[0] + q.begin + jj);
                 float w = wp[jj];
                 float m = HM ? mp[jj] : 0.f;
                 const float cj = use_se ? __ldcs(ptr[3] + q.begin + jj) : (PE ? 1.f : ct);
-                if (SW) aw = __fmaf_rn(w, w, aw);
+                if (SW) awt = __fma_rn((double)w, (double)w, awt);
                 sgd1(g, cj, w, m, sc, HM);
                 wp[jj] = w;
                 if (HM) mp[jj] = m;
             }
-            ptile[p] = tab.c0 + c;
-            pend[p] = aw;
+            if (SW) {
+                if (tile_tail) {
+                    store_w_tile_now(sc.part2 + tab.c0 + c, aw, ew, awt);
+                } else {
+                    ptile[p] = tab.c0 + c;
+                    pend[p] = aw;
+                    if (ew) ecode |= scale_code(ew) << (2 * p);
+                }
+            }
         }
         if (SW) {
-            warp_sums<kPend>(pend);
-            if (lane == 0) {
-#pragma unroll
-                for (int p = 0; p < kPend; ++p)
-                    if (ptile[p] >= 0)
-                        st_keep_l2(sc.part2 + ptile[p], make_float2(pend[p], 0.f),
-                                   policy_evict_last());
+            // reduce-scatter: lanes 8p hold tile p's total
+            int idx;
+            const float f = warp_reduce_scatter<kPend>(pend, idx);
+            if ((lane & 7) == 0) {
+                const int t = idx == 0 ? ptile[0] : idx == 1 ? ptile[1] : idx == 2 ? ptile[2] : ptile[3];
+                if (t >= 0)
+                    st_keep_l2(sc.part2 + t,
+                               widen_scaled(f, -2 * scale_exp((ecode >> (2 * idx)) & 3u)),
+                               policy_evict_last());
             }
         }
         if (stop) break;
@@ -1522,10 +1700,10 @@ WsLayout ws_layout(int n_tensors, const Plan &pl) {
     L.tiles = take(sizeof(unsigned) * 4);
     L.sctr1 = take(sizeof(unsigned) * (size_t)n_tensors);
     L.sctr2 = take(sizeof(unsigned) * (size_t)n_tensors);
-    L.part1 = take(sizeof(float2) * kAcc * (size_t)pl.c1);
-    L.part2 = take(sizeof(float2) * (size_t)pl.c2);
-    L.spart1 = take(sizeof(float2) * kAcc * (size_t)pl.s1);
-    L.spart2 = take(sizeof(float2) * (size_t)pl.s2);
+    L.part1 = take(sizeof(double) * kAcc * (size_t)pl.c1);
+    L.part2 = take(sizeof(double) * (size_t)pl.c2);
+    L.spart1 = take(sizeof(double) * kAcc * (size_t)pl.s1);
+    L.spart2 = take(sizeof(double) * (size_t)pl.s2);
     L.tsum = take(sizeof(double) * kTsum * (size_t)n_tensors);
     L.cand = take(sizeof(float) * (size_t)n_tensors);
     L.total = off;
@@ -1667,7 +1845,7 @@ int launch_streaming(Kernel kernel, int n, const int64_t *numels, int chunk, int
 }
 
 // k_combine over all tensors (tiles of `chunk` elements), NA sums per tile.
-template <int NA, bool PREC>
+template <int NA>
 int launch_combine(int n, const int64_t *numels, int chunk, const Scalars &sc_in, cudaStream_t s) {
     std::unique_ptr<CombTable> tab(new CombTable);
     Scalars sc = sc_in;
@@ -1700,7 +1878,7 @@ int launch_combine(int n, const int64_t *numels, int chunk, const Scalars &sc_in
         tab->sfirst[cnt] = ns;
         s_global += ns;
         const int grid = (ns + kCombWarps - 1) / kCombWarps;
-        const int rc = launch_pdl(k_combine<NA, PREC>, grid, 32 * kCombWarps, 0, s, *tab, sc);
+        const int rc = launch_pdl(k_combine<NA>, grid, 32 * kCombWarps, 0, s, *tab, sc);
         if (rc) return rc;
     }
     return TULA_OK;
@@ -1737,10 +1915,10 @@ Scalars make_scalars(const tula_ags_hparams *hp, int K, int n, void *ws, const W
     sc.tiles = reinterpret_cast<unsigned *>(b + L.tiles);
     sc.sctr1 = reinterpret_cast<unsigned *>(b + L.sctr1);
     sc.sctr2 = reinterpret_cast<unsigned *>(b + L.sctr2);
-    sc.part1 = reinterpret_cast<float2 *>(b + L.part1);
-    sc.part2 = reinterpret_cast<float2 *>(b + L.part2);
-    sc.spart1 = reinterpret_cast<float2 *>(b + L.spart1);
-    sc.spart2 = reinterpret_cast<float2 *>(b + L.spart2);
+    sc.part1 = reinterpret_cast<double *>(b + L.part1);
+    sc.part2 = reinterpret_cast<double *>(b + L.part2);
+    sc.spart1 = reinterpret_cast<double *>(b + L.spart1);
+    sc.spart2 = reinterpret_cast<double *>(b + L.spart2);
     sc.tsum = reinterpret_cast<double *>(b + L.tsum);
     sc.cand = reinterpret_cast<float *>(b + L.cand);
     return sc;
@@ -1760,7 +1938,7 @@ int run_reduce_k(int K, int n, const int64_t *numels, const Scalars &sc, int gri
                                           grid, s, fill);
     if (rc) return rc;
     record(mid_event, s);
-    return launch_combine<kAcc, PR>(n, numels, chunk, sc, s);
+    return launch_combine<kAcc>(n, numels, chunk, sc, s);
 }
 
 template <bool WM, bool RW, bool SS, bool PR, typename Fill>
@@ -1975,7 +2153,7 @@ int run_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mo
 #undef TULA_UPD
     if (rc) return rc;
     record(hp->trace_events[3], s);
-    if (sw) rc = launch_combine<1, false>(n, numels, c2, sc, s);
+    if (sw) rc = launch_combine<1>(n, numels, c2, sc, s);
     if (rc) return rc;
     record(hp->trace_events[4], s);
     return TULA_OK;

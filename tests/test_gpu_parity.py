@@ -462,3 +462,59 @@ def test_update_scale_over_the_whole_float_range():
     O.update_scale(W.to_numpy(gs), W.to_numpy(gl), hp.eps, 1e30, O.GRAN_TENSOR, scale=ref)
     torch.cuda.synchronize()
     assert_norm_close(scale.cpu().numpy(), ref, "scale", rtol=2.0 ** -22)
+
+
+def _scale_weights(pair, seed, lo=1e-24, hi=1e22):
+    """Multiplies each tensor's w by its own factor, the factors evenly spaced in log from lo to
+    hi and shuffled, on both sides (the same fp32 products), so that weight squares underflow,
+    overflow and stay ordinary."""
+    rng = np.random.default_rng([seed, 9])
+    f = np.exp(rng.permutation(np.linspace(math.log(lo), math.log(hi), pair.n))).astype(np.float32)
+    assert (f < 1e-20).any() and (f > 1e20).any()
+    for p, t in enumerate(pair.buf.w):
+        t.mul_(float(f[p]))
+    torch.cuda.synchronize()
+    pair.w_h = W.to_numpy(pair.buf.w)
+
+
+def test_default_steps_over_the_whole_float_range():
+    """Algorithm 1 steps on the default path (fp32 sums within a tile, no refresh, no LARS) and
+    tula_layer_stats, with gradient and weight factors from 1e-24 to 1e22: tiles whose fp32
+    sums of squares would overflow, underflow, or hold only zeros are summed again with an exact
+    power-of-two scaling; norms, |G|^2, Delta, the branch, w and m match the oracle."""
+    ps = _extreme_pset(2)
+    wl = _extreme_workload(113, ps)
+    pair = Pair(wl, K=2, pset=ps)
+    _scale_weights(pair, 113)
+    rng = np.random.default_rng(114)
+    s0 = rng.uniform(0.5, 2.0, size=pair.n).astype(np.float32)   # a non-trivial gradscale
+    pair.gpu.scale.copy_(torch.from_numpy(s0))
+    pair.scale_h = s0.copy()
+    # unscaled (first step), scaled (Delta = 0), unscaled (x2: Delta = 3)
+    for seed_step, mult in ((1, 1.0), (1, 1.0), (1, 2.0)):
+        pair.step(seed_step, mult)
+    assert pair.flags == [0, 1, 0]
+    # the statistics alone, read-only, over the same range
+    W.fill_grads(pair.buf, wl, step=2)
+    stats = torch.zeros(pair.n, T.TULA_STATS_LEN, dtype=torch.float64, device="cuda")
+    T.tula_layer_stats(pair.buf.w, pair.buf.g, stats, pair.gpu.workspace)
+    ref = O.layer_stats(W.to_numpy(pair.buf.w), [W.to_numpy(pair.buf.g[k]) for k in range(2)])
+    torch.cuda.synchronize()
+    assert_stats_close(stats.cpu().numpy(), ref, "layer_stats over the whole float range")
+    big = ref[:, T.TULA_STAT_W_SQ] > 3.4e38
+    tiny = (ref[:, T.TULA_STAT_G_SQ] > 0) & (ref[:, T.TULA_STAT_G_SQ] < 1e-38)
+    assert big.any() and tiny.any()  # the case is what it claims to be
+
+
+@pytest.mark.parametrize("K", [1, 4])
+def test_default_steps_misaligned_over_the_whole_float_range(K):
+    """The same range on misaligned tensors, where every element is loaded one by one (fp64
+    squares), and with K = 1 and 4 (other tile sizes and stream counts)."""
+    ps = _extreme_pset(K if K > 1 else 1)
+    wl = _extreme_workload(121 + K, ps)
+    for shift in (0, 1):
+        pair = Pair(wl, K=K, pset=ps, align=1 if shift else 64, shift=shift)
+        _scale_weights(pair, 121 + K)
+        pair.step(1, 1.0)
+        pair.step(1, 1.0)
+        assert pair.flags == [0, 1]
