@@ -35,15 +35,17 @@
  *     step may be partly applied: zero the workspace again before reusing it.
  *   - Element-wise arithmetic is IEEE fp32, one rounding per operation, in the
  *     order written below (no fused multiply-add).  Squared norms are fp32 sums
- *     within a tile (<= 8192 elements; relative error below ~4e-6) added across
- *     tiles in fp64.  A tile whose fp32 sums would overflow (a lane sum above
+ *     within a tile (<= 9216 elements; relative error below ~4e-6) added across
+ *     tiles exactly, in integers (fixed point from 2^-352 to 2^320, by L2
+ *     atomics, so the order tiles land in cannot change a bit), then rounded
+ *     once to fp64.  A tile whose fp32 sums would overflow (a lane sum above
  *     2^120) or lose precision to underflow (every lane sum below 2^-100, zero
  *     included) is summed again with its elements scaled by an exact power of two,
  *     and elements loaded one by one (tails, misaligned tensors) are squared in
  *     fp64, so these norms hold over the whole fp32 range.  Norms that feed a
  *     coefficient (gradscale refresh, LARS) split every square exactly into two
  *     fp32 parts, add them as float-float pairs per lane and in fp64 across lanes
- *     and tiles (relative error ~1e-14); a tile whose pairs cannot hold that (a
+ *     (relative error ~1e-14), then exactly across tiles; a tile whose pairs cannot hold that (a
  *     square that overflows, or sums below 2^-77) is redone with exact fp64
  *     squares, so these norms keep that precision over the whole fp32 range.
  */
@@ -135,11 +137,12 @@ typedef struct tula_ags_hparams {
                                      not depend on it) */
     void *trace_events[5];        /* optional cudaEvent_t (NULL = none), recorded on `stream`:
                                      [0] before the reduction kernel(s), [1] after them,
-                                     [2] after the pass-1 combine (before the update kernel),
-                                     [3] after the update kernel(s), [4] after the pass-2
-                                     combine (the end of the step).  A recorded event keeps the
-                                     next kernel from starting early, so steps that record
-                                     events run slightly slower. */
+                                     [2] before the update kernel(s) (after a finish kernel
+                                     between the passes, which only LARS and per-element steps
+                                     have), [3] after the update kernel(s), [4] the end of the
+                                     step (after its last finish kernel).  A recorded event
+                                     keeps the next kernel from starting early, so steps that
+                                     record events run slightly slower. */
 } tula_ags_hparams;
 
 /* Fills *hp with the paper's defaults for K replicas: AGS, per tensor, automatic branch,
@@ -147,7 +150,8 @@ typedef struct tula_ags_hparams {
  * static_s 1, lars_trust 1; all pointers NULL, grid_ctas 0. */
 void tula_ags_default_hparams(tula_ags_hparams *hp, int K);
 
-/* Bytes of workspace needed for this list of tensor sizes and K replicas (host only). */
+/* Bytes of workspace needed for this list of tensor sizes and K replicas (host only): about
+ * 3.1 KB per tensor (accumulators and per-tensor sums), whatever the tensors' sizes. */
 int tula_ags_workspace_size(const int64_t *numels, int n_tensors, int K, size_t *bytes);
 
 /*
@@ -158,11 +162,12 @@ int tula_ags_workspace_size(const int64_t *numels, int n_tensors, int K, size_t 
  *                          the other replicas are only read
  *   mom_ptrs[p]            momentum buffer m_p, device fp32, updated in place; mom_ptrs may be
  *                          NULL only when momentum == 0 (then w <- w - lr * d)
- *   numels[p] >= 0         element counts (0 = skipped); one tensor may span at most
- *                          1,694,208 tiles of min(tula_ags_chunk_elems(1, K + 1),
+ *   numels[p] >= 0         element counts (0 = skipped); all tensors together may span
+ *                          fewer than 2^31 tiles of min(tula_ags_chunk_elems(1, K + 1),
  *                          tula_ags_chunk_elems(2, 4)) elements (K + 2 in place of K + 1
- *                          when K = 1): about 2.6e9 elements for K <= 4, 1.5e9 at K = 8,
- *                          6.5e8 at K = 16; a larger tensor gives TULA_ERR_ARG
+ *                          when K = 1; an empty tensor counts as one tile): about 3.3e12
+ *                          elements for K <= 4, 1.9e12 at K = 8, 8.2e11 at K = 16, more
+ *                          than any GB300 holds; a longer list gives TULA_ERR_ARG
  * Per element, with c the coefficient of the rule (Algorithm 1, Eq. 8):
  *   gbar = (((g_0 + g_1) + ...) + g_{K-1}) / K
  *   d    = c * gbar + weight_decay * w
@@ -214,10 +219,9 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
  * TULA_STATIC_SCRATCH_BYTES (16 MiB) inside this library.  Every GPU that loads the library holds
  * that array until the process exits.  hp->workspace and hp->workspace_bytes are ignored.
  *
- * Limit: the scratch a tensor list needs (tula_ags_workspace_size) is about 110 bytes per tensor
- * plus, per 1000 parameters, 14 bytes (K <= 2), 21 (K = 4), 32 (K = 8) or 68 (K = 16): e.g. 4096
- * tensors holding up to ~1.2e9 parameters at K <= 2, ~5.1e8 at K = 8, ~2.4e8 at K = 16.  A larger
- * list is rejected with TULA_ERR_SCRATCH_LIMIT before anything is enqueued.
+ * Limit: the scratch a tensor list needs (tula_ags_workspace_size) is about 3.1 KB per tensor,
+ * whatever the tensors' sizes and K: up to 5,397 tensors.  A longer list is rejected with
+ * TULA_ERR_SCRATCH_LIMIT before anything is enqueued.
  *
  * Set-up: every call looks up the array's device address in the current device's context
  * (cudaGetSymbolAddress, a host-side lookup), so the address never goes stale, also after
@@ -267,7 +271,7 @@ uint64_t tula_ags_launch_count(void);
 
 /*
  * Elements per tile (work item) of a pass that streams `streams` tensors through shared memory:
- * pass 1, the reduction (K replicas [+ w] [+ g_small]; one tile of every stream fills a 32 KB
+ * pass 1, the reduction (K replicas [+ w] [+ g_small]; one tile of every stream fills a 36 KB
  * stage), or pass 2, the update (gbar, w [+ m] [+ per-element scale]; a 24 KB stage).  A multiple
  * of 128; TULA_ERR_ARG for another pass or when streams is outside [1, TULA_MAX_K + 2] (pass 1)
  * or [1, 4] (pass 2).

@@ -4,21 +4,23 @@
 // dependent launch so that each one's launch and prologue overlap the tail of
 // the one before:
 //
-//   k_reduce   (pass 1)  K-way replica mean (Eq. 1c) written over replica 0, and
-//                        per-tile partial sums of |gbar|^2, |g_0|^2 [, |w|^2].
-//   k_combine            per tensor, the fixed-order sum of its tile partials,
-//                        its statistics, its coefficient when scaled (the old
+//   k_reduce   (pass 1)  K-way replica mean (Eq. 1c) written over replica 0; each
+//                        tile's sums of |gbar|^2, |g_0|^2 [, |w|^2] are added
+//                        exactly into per-tensor accumulators (and |gbar|^2 into
+//                        the step's |G|^2 accumulator) by L2 atomics.
+//   k_finish             per tensor, the norms rounded from its accumulators, its
+//                        statistics, its coefficient when scaled (the old
 //                        gradscale, Eq. 8's s, or the LARS ratio) and, when
 //                        asked, the refreshed gradscale (UpdateGradScale,
-//                        Algorithm 1); the warp taking the last segment ticket
-//                        forms |G|^2, Delta (Eq. 5) and the branch of Algorithm 1.
+//                        Algorithm 1); one more warp forms |G|^2, Delta (Eq. 5)
+//                        and the branch of Algorithm 1.
 //   k_update   (pass 2)  d = c gbar + wd w; m = mu m + d; w = w - lr m (Eq. 7b with
 //                        the wrapped SGD); |w|^2 per tile for the statistics,
-//   k_combine            then summed per tensor.
+//   k_finish             then rounded per tensor.
 //
 // The streaming passes: each tensor is cut into tiles of T elements (T fixed
 // per pass by how many tensors it streams, so that one tile of every stream
-// fills one shared-memory stage: 32 KB in pass 1, 24 KB in pass 2).  One
+// fills one shared-memory stage: 36 KB in pass 1, 24 KB in pass 2).  One
 // persistent CTA per SM; small launches deal tiles round-robin, larger ones
 // claim them from a global counter (SMs stream at unequal rates).  The producer
 // warp moves tiles from HBM into the stage ring with TMA bulk copies
@@ -26,8 +28,8 @@
 // lane each; consumer warps, each owning whole stages, compute from shared
 // memory and release the stage through an mbarrier.  Tile partials are fp32
 // sums within a tile (float-float pairs per lane in the precise mode for norms
-// that feed a coefficient), range-checked per tile and stored as fp64; only
-// plain stores leave a tile.
+// that feed a coefficient), range-checked per tile, and leave the tile only as
+// exact integer additions into the accumulators.
 //
 // Every mbarrier wait is bounded; a wait that runs out sets an error word in
 // the workspace (tula_ags_workspace_error) and the CTA drains its copies in
@@ -35,9 +37,9 @@
 // 20-70 bytes); nothing here is a contraction, so no tensor cores.  The tile
 // table, pointers and sizes travel in the kernel parameter block
 // (__grid_constant__, up to ~31 KB per launch): no host-to-device copy,
-// allocation or host sync is ever needed.  Each tile's partials go to the
-// tile's own slot and are summed in an order fixed by the numels, so results
-// are bitwise reproducible and independent of the grid.
+// allocation or host sync is ever needed.  Integer addition does not depend on
+// the order in which tiles land, so results are bitwise reproducible and
+// independent of the grid and of which CTA took which tile.
 #include "tula_ags.h"
 
 #include <cuda_runtime.h>
@@ -77,10 +79,10 @@ struct Ring {
 // Pass 1 streams K (+1, +2) tensors and little arithmetic: large copies, few
 // consumers.  Pass 2 does ~11 flops per element over 3-4 streams: its
 // consumers, not HBM, set the pace with three warps, so it runs four.
-using Ring1 = Ring<32, 6, 3>;
+using Ring1 = Ring<36, 6, 3>;
 // The precise pass 1 (float-float squares) spends ~13 dependent FP32 instructions per element
 // and norm: six consumers, two per scheduler, hide that latency.  Same stages, same tiles.
-using Ring1P = Ring<32, 6, 6>;
+using Ring1P = Ring<36, 6, 6>;
 template <bool PR>
 using Ring1For = std::conditional_t<PR, Ring1P, Ring1>;
 static_assert(Ring1P::kStageBytes == Ring1::kStageBytes && Ring1P::kStages == Ring1::kStages,
@@ -90,8 +92,7 @@ constexpr int kDynTiles = 64;            // tiles per CTA from which a launch cl
 constexpr unsigned kClaim = 4;           // tiles per claim
 constexpr unsigned kClaimTail = 16;      // single-tile claims for the last kClaimTail per CTA
 constexpr int kPend = 4;                // tiles whose warp reductions run together
-constexpr int kCombWarps = 4;           // k_combine: one warp per segment, 4 per CTA
-constexpr int kSegTiles = 256;          // tile partials per combine segment (8 per lane)
+constexpr int kFinWarps = 4;            // k_finish: one warp per tensor, 4 per CTA
 constexpr int kParamBudget = 31 * 1024; // kernel parameter bytes per launch (limit 32764)
 constexpr int kAcc = 3;                 // partial sums per pass-1 tile: |gbar|^2, |g_0|^2, |w|^2
 constexpr int kPrecCols = 1;            // float4 columns per step of the precise path's tile loop
@@ -121,41 +122,21 @@ struct Table {
     const float *ptr[kMaxT][NP];
 };
 
-// k_combine: where each tensor's tile partials are, cut into segments of at
-// most kSegTiles tiles.
-struct CombTable {
-    static constexpr int kMaxT = 1536;
-    static constexpr int kMaxS = (kParamBudget - 64 - 12 * (kMaxT + 1)) / 2;
-    int n;   // tensors in this launch
-    int t0;  // global index of its first tensor
-    int s0;  // global index of its first segment
-    int ns;  // segments in this launch
-    int cfirst[kMaxT];          // global index of the tensor's first tile
-    int ntiles[kMaxT];          // its tile count
-    int sfirst[kMaxT + 1];      // its first segment, relative to s0; sfirst[n] = ns
-    unsigned short seg_t[kMaxS];  // the tensor (index in this launch) of each segment
-};
-
 struct Scalars {
     int K, rule, gran, force, refresh, mode, n_total, read_w;
-    int pow2K, evict_first, n_seg1, pad2;  // evict_first: TMA loads ask L2 to drop their lines
-                                           // first; n_seg1: combine segments of pass 1
+    int pow2K, evict_first, pad1, pad2;  // evict_first: TMA loads ask L2 to drop their lines first
     float delta, eps, s_max, static_s, lars_trust, lr, mu, wd, invK, Kf;
     float *scale;
     double *state;
     double *stats;
-    unsigned *done;  // [1]: segments combined in a step (the branch's ticket)
-    int *flags;      // [0]: branch of the last step (1 = scaled)
-    unsigned *err;   // [0]: bounded waits that ran out (sticky until read)
-    unsigned *sctr1; // [tensor]: segments combined, pass 1
-    unsigned *sctr2; // [tensor]: segments combined, pass 2
-    double *part1;   // [tile][kAcc], pass 1
-    double *part2;   // [tile], pass 2 (|w|^2)
-    double *spart1;  // [segment][kAcc], pass 1
-    double *spart2;  // [segment], pass 2
-    double *tsum;    // [tensor][kTsum]: |gbar|^2, |g_0|^2, |w|^2
-    float *cand;     // [tensor]: c_p of the scaled branch (AGS: the old gradscale)
-    unsigned *tiles; // [2 * pass]: next tile to claim, [2 * pass + 1]: CTAs finished
+    int *flags;                // [0]: branch of the last step (1 = scaled)
+    unsigned *err;             // [0]: bounded waits that ran out (sticky until read)
+    unsigned long long *acc1;  // [tensor][kAcc][kTCopies][kAccWords]: |gbar|^2, |g_0|^2, |w|^2
+    unsigned long long *gacc;  // [kGCopies][kAccWords]: |G|^2 = every tensor's |gbar|^2
+    unsigned long long *acc2;  // [tensor][kTCopies][kAccWords]: |w|^2, pass 2
+    double *tsum;              // [tensor][kTsum]: |gbar|^2, |g_0|^2, |w|^2
+    float *cand;               // [tensor]: c_p of the scaled branch (AGS: the old gradscale)
+    unsigned *tiles;           // [2 * pass]: next tile to claim, [2 * pass + 1]: CTAs finished
 };
 
 // ----------------------------------------------------------------------------
@@ -167,16 +148,6 @@ __device__ __forceinline__ void st_stream(float *p, float4 v) {
 }
 __device__ __forceinline__ void st_keep(float *p, float4 v) {
     *reinterpret_cast<float4 *>(p) = v;
-}
-// 8-byte store that asks L2 to keep the line: tile partials, read back by the
-// combine kernel right after the streaming kernel that writes them.
-__device__ __forceinline__ void st_keep_l2(double *p, double v, uint64_t policy) {
-    asm volatile("st.global.L2::cache_hint.f64 [%0], %1, %2;" ::"l"(p), "d"(v), "l"(policy) : "memory");
-}
-__device__ __forceinline__ uint64_t policy_evict_last() {
-    uint64_t p;
-    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-    return p;
 }
 // 16-byte load from shared memory (a shared-window address).
 __device__ __forceinline__ float4 lds4(uint32_t addr) {
@@ -343,9 +314,6 @@ __device__ __forceinline__ bool dw_lane_ok(float2 v) {
 
 // Exact powers of two (k within the normal range of the type).
 __device__ __forceinline__ float pow2f(int k) { return __int_as_float((k + 127) << 23); }
-__device__ __forceinline__ double pow2d(int k) {
-    return __longlong_as_double((long long)(k + 1023) << 52);
-}
 
 // Range of a tile's fp32 sums of squares, decided for the whole warp from the largest lane
 // sum v (>= 0, or NaN): 0 when every lane sum is safe as it stands, else the exponent e of a
@@ -354,9 +322,9 @@ __device__ __forceinline__ double pow2d(int k) {
 //    sums that fell below fp32's normal range err by at most 2^-150 each, < 2^-38 of the tile
 //    sum: kept.
 //  * max above 2^120, inf or NaN: a square or a sum reached fp32's top.  Scaled by 2^-72 every
-//    finite element is below 2^56, its square below 2^112, a lane's sum of up to 256 squares
-//    below 2^120; what the scaling pushes below 2^-149 has a square under 2^-254 of the tile
-//    sum.  Inf and NaN stay inf and NaN.
+//    finite element is below 2^56, its square below 2^112, a lane's sum of up to 288 squares
+//    below 2^121 and the tile's below 2^126; what the scaling pushes below 2^-149 has a square
+//    under 2^-254 of the tile sum.  Inf and NaN stay inf and NaN.
 //  * max below 2^-100 (zero included): every element is below 2^-50 in magnitude (a sum of
 //    squares is at least its largest term), so 2^100 x is exact, below 2^50, and its square is a
 //    normal number unless x is 0.
@@ -375,20 +343,140 @@ __device__ __forceinline__ int sq_range_exp(float v) {
     if (m < __float_as_uint(0x1p-100f)) return kScaleUp;
     return 0;
 }
-// x * 2^k as a double, exactly, built on the integer pipes (GB300's FP64 pipe is slow): x is a
-// tile's range-checked fp32 sum, i.e. zero, normal, inf or NaN; a subnormal x (which the range
-// check rules out) takes the fp64 route.
-__device__ __forceinline__ double widen_scaled(float x, int k) {
-    const unsigned u = __float_as_uint(x);
-    const unsigned e = (u >> 23) & 0xffu;
-    const unsigned long long sign = (unsigned long long)(u >> 31) << 63;
-    const unsigned long long man = (unsigned long long)(u & 0x7fffffu) << 29;
-    if (e == 0u) return man ? __dmul_rn((double)x, pow2d(k)) : __longlong_as_double((long long)sign);
-    const unsigned long long ex = e == 0xffu ? 0x7ffull : (unsigned long long)((int)e - 127 + 1023 + k);
-    return __longlong_as_double((long long)(sign | (ex << 52) | man));
-}
 __device__ __forceinline__ float4 mul4(float4 v, float f) {
     return make_float4(__fmul_rn(v.x, f), __fmul_rn(v.y, f), __fmul_rn(v.z, f), __fmul_rn(v.w, f));
+}
+
+// ----------------------------------------------------------------------------
+// Exact accumulation of the squared norms
+// ----------------------------------------------------------------------------
+//
+// The partial sums of squares (one per tile and norm, all >= 0) are added up exactly, in
+// integers: an accumulator is a fixed-point number of kAccDigits 32-bit digits, digit i of
+// weight 2^(32 i + kAccBase), each held in the low half of a 64-bit word whose high half
+// collects carries.  A partial m * 2^E (m an fp32 or fp64 significand) touches two or three
+// consecutive words, each by an atomic add that nothing waits for (red.global.add.u64).
+// Integer addition is associative, so the sum does not depend on the order the tiles land in:
+// norms are bitwise reproducible for any grid and any claim order, and they are the exact sums
+// of the tile partials, rounded once to fp64 when read (acc_to_double).
+//
+// Range: the partials are fp32 tile sums scaled by 2^k (k in {0, -200, 144}, sq_range_exp) or
+// fp64 sums of exact squares of fp32 numbers, so their bits lie within 2^-352 .. 2^273; a tensor
+// of up to 2^31 tiles, or all tensors together, stays below 2^305; 21 digits from 2^-352 cover
+// 2^-352 .. 2^320.  Each word takes at most two adds (< 2^32 each) per tile, so its high half
+// cannot overflow for fewer than 2^31 tiles.  A partial that is inf or NaN (an inf or NaN
+// element) sets a flag in the last word instead: the norm is then inf, or NaN.
+//
+// Copies: the tiles of one tensor land close together in time, and every tile of a step adds
+// into |G|^2, so one word would take an atomic every few ns, about what an L2 slice can do for
+// one address.  Each accumulator therefore has copies, picked by the CTA, that the reading warp
+// adds up (exact; all copies together still take fewer than 2^32 adds per word).
+constexpr int kAccDigits = 21;
+constexpr int kAccWords = 24;             // digits, two spare words, the flags
+constexpr int kAccFlags = kAccWords - 1;  // bit 0: an inf partial, bit 1: a NaN partial
+constexpr int kAccBase = -352;
+constexpr int kTCopies = 4;               // copies of each per-tensor accumulator
+constexpr int kGCopies = 8;               // copies of the |G|^2 accumulator
+static_assert(kAccDigits <= kAccFlags && kAccWords <= 32, "one word per lane");
+static_assert((kTCopies & (kTCopies - 1)) == 0 && (kGCopies & (kGCopies - 1)) == 0, "powers of 2");
+
+// Adds m * 2^E (m < 2^53, kAccBase <= E, E + 53 <= 2^32 weight of the top digit) to A.
+__device__ __forceinline__ void acc_add(unsigned long long *A, unsigned long long m, int E) {
+    if (m == 0ull) return;
+    const int s = E - kAccBase;
+    const int i = s >> 5, r = s & 31;
+    const unsigned long long lo = m << r;
+    const unsigned long long hi = r ? (m >> (64 - r)) : 0ull;
+    if (lo & 0xffffffffull) atomicAdd(A + i, lo & 0xffffffffull);
+    if (lo >> 32) atomicAdd(A + i + 1, lo >> 32);
+    if (hi) atomicAdd(A + i + 2, hi);
+}
+// Adds f * 2^k for an fp32 f >= 0 (or inf, NaN).
+__device__ __forceinline__ void acc_add_f32(unsigned long long *A, float f, int k) {
+    const unsigned u = __float_as_uint(f);
+    const unsigned e = (u >> 23) & 0xffu;
+    if (e == 0xffu) {
+        atomicOr(A + kAccFlags, (u & 0x7fffffu) ? 2ull : 1ull);
+        return;
+    }
+    const unsigned long long m = e ? ((u & 0x7fffffu) | 0x800000u) : (u & 0x7fffffu);
+    acc_add(A, m, (e ? (int)e : 1) - 150 + k);
+}
+// Adds an fp64 d >= 0 (or inf, NaN).
+__device__ __forceinline__ void acc_add_f64(unsigned long long *A, double d) {
+    const unsigned long long u = (unsigned long long)__double_as_longlong(d);
+    const unsigned e = (unsigned)(u >> 52) & 0x7ffu;
+    const unsigned long long f = u & 0xfffffffffffffull;
+    if (e == 0x7ffu) {
+        atomicOr(A + kAccFlags, f ? 2ull : 1ull);
+        return;
+    }
+    acc_add(A, e ? (f | (1ull << 52)) : f, (e ? (int)e : 1) - 1075);
+}
+
+// The values of R accumulators rounded to the nearest double (ties to even), by the whole
+// warp: lane i passes word i of each (any value for lanes >= kAccWords).  Carries first move up
+// one word (each high half, < 2^32, into the next digit), which leaves at most one carry per
+// digit; those ripple through runs of all-ones digits, found for all 32 digits at once with two
+// votes and one integer addition (the carry-lookahead of an adder).  Then the top three digits
+// give the 53-bit significand, its round bit and, with every digit below, its sticky bit.  The
+// R conversions go stage by stage together, so their shuffle and vote latencies overlap.
+template <int R>
+__device__ __forceinline__ void acc_to_double(const unsigned long long (&wi)[R], double (&out)[R]) {
+    const int lane = threadIdx.x & 31;
+    unsigned long long flags[R], v[R];
+    unsigned d[R], nz[R];
+#pragma unroll
+    for (int r = 0; r < R; ++r) flags[r] = __shfl_sync(kFull, wi[r], kAccFlags);
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const unsigned long long w = lane < kAccDigits ? wi[r] : 0ull;
+        const unsigned long long up = __shfl_up_sync(kFull, w >> 32, 1);
+        v[r] = (w & 0xffffffffull) + (lane > 0 ? up : 0ull);  // < 2^33
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const unsigned G = __ballot_sync(kFull, (v[r] >> 32) != 0ull);
+        const unsigned P = __ballot_sync(kFull, (v[r] & 0xffffffffull) == 0xffffffffull);
+        const unsigned carries = ((G | P) + G) ^ (G | P) ^ G;  // bit i: a carry into digit i
+        d[r] = (unsigned)(v[r] + ((carries >> lane) & 1u));
+    }
+#pragma unroll
+    for (int r = 0; r < R; ++r) nz[r] = __ballot_sync(kFull, d[r] != 0u);
+#pragma unroll
+    for (int r = 0; r < R; ++r) {
+        const int top = nz[r] ? 31 - __clz(nz[r]) : 0;
+        const unsigned d0 = __shfl_sync(kFull, d[r], top);
+        const unsigned d1 = __shfl_sync(kFull, d[r], top > 0 ? top - 1 : 0);
+        const unsigned d2 = __shfl_sync(kFull, d[r], top > 1 ? top - 2 : 0);
+        if (flags[r] & 2ull) {
+            out[r] = __longlong_as_double(0x7ff8000000000000ll);  // NaN
+        } else if (flags[r] & 1ull) {
+            out[r] = __longlong_as_double(0x7ff0000000000000ll);  // +inf
+        } else if (nz[r] == 0u) {
+            out[r] = 0.0;
+        } else {
+            const unsigned m1 = top > 0 ? d1 : 0u, m2 = top > 1 ? d2 : 0u;
+            const bool below = top > 2 && (nz[r] & ((1u << (top - 2)) - 1u)) != 0u;
+            const int L = 32 - __clz(d0);  // bit length of the top digit
+            const int z = 32 - L;          // shift that puts its leading 1 at bit 63
+            const unsigned long long hi = ((unsigned long long)d0 << 32) | m1;
+            const unsigned long long T = (hi << z) | (z ? ((unsigned long long)m2 >> (32 - z)) : 0ull);
+            const bool rest = (m2 & (0xffffffffu >> z)) != 0u;  // bits of m2 below T
+            unsigned long long mant = T >> 11;
+            const bool round = (T >> 10) & 1ull;
+            const bool sticky = (T & 0x3ffull) != 0ull || rest || below;
+            int ex = 32 * top + kAccBase + L - 1;  // weight of the leading bit
+            if (round && (sticky || (mant & 1ull))) {
+                if (++mant == (1ull << 53)) {
+                    mant >>= 1;
+                    ++ex;
+                }
+            }
+            out[r] = __longlong_as_double(
+                (long long)(((unsigned long long)(ex + 1023) << 52) | (mant & 0xfffffffffffffull)));
+        }
+    }
 }
 
 // ----------------------------------------------------------------------------
@@ -468,14 +556,6 @@ __device__ __forceinline__ uint64_t policy_evict_first() {
     return p;
 }
 
-// Ticket counter increment with acquire-release semantics at GPU scope: the
-// caller's earlier stores are visible to whoever later takes the last ticket.
-__device__ __forceinline__ unsigned ticket(unsigned *ctr) {
-    unsigned r;
-    asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], 1;" : "=r"(r) : "l"(ctr) : "memory");
-    return r;
-}
-__device__ __forceinline__ void fence_acq_rel() { asm volatile("fence.acq_rel.gpu;" ::: "memory"); }
 
 __device__ __forceinline__ void report_timeout(const Scalars &sc) {
     atomicOr(sc.err, 1u);
@@ -581,7 +661,7 @@ struct TensorCache {
 //    launch end with the memory system rather than with its slowest SM.  The
 //    last CTA to finish puts both counters (ctr[0], ctr[1]) back to zero.
 // Where a tile is processed never changes its result: each tile's partial sums
-// go to the tile's own slot and are combined in a fixed order later.  The j-th
+// are added exactly, in integers, into its tensor's accumulators.  The j-th
 // tile of a CTA goes to stage j % kStages and is consumed by consumer warp
 // j % kConsumers; its launch tile index is left in stage_tile[stage] before the
 // stage's full barrier is armed (the barrier's release/acquire orders it), and
@@ -746,7 +826,8 @@ __device__ __forceinline__ int next_tile(const Scalars &sc, int j, uint64_t *ful
 // norms that feed a per-tensor coefficient (UpdateGradScale, LARS).  Otherwise the tile's sum
 // stays in fp32: each lane adds <= 16 squares per group of 4 columns, then the
 // group sums, then a 5-level tree across lanes, a relative error below 71 ulp
-// (4e-6) of the tile's sum; tiles are combined in fp64.  That is what the
+// (4e-6) of the tile's sum; tiles are added exactly into the tensor's
+// accumulator.  That is what the
 // variability metric and the statistics need, and it keeps GB300's slow FP64
 // pipe out of the streaming loop.  One warp vote per tile (sq_range_exp) keeps
 // it valid over the whole fp32 range: a tile whose fp32 sums would overflow or
@@ -1006,12 +1087,23 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
 
 static_assert(kPend == 4, "the owner lanes below pick one of four tiles");
 
+// This CTA's copies of the accumulators: tensor tg's pass-1 norm a, |G|^2, tensor tg's |w|^2
+// in pass 2.
+__device__ __forceinline__ unsigned long long *acc1_of(const Scalars &sc, int tg, int a) {
+    return sc.acc1 + (((size_t)tg * kAcc + a) * kTCopies + (blockIdx.x & (kTCopies - 1))) * kAccWords;
+}
+__device__ __forceinline__ unsigned long long *gacc_of(const Scalars &sc) {
+    return sc.gacc + (size_t)(blockIdx.x & (kGCopies - 1)) * kAccWords;
+}
+__device__ __forceinline__ unsigned long long *acc2_of(const Scalars &sc, int tg) {
+    return sc.acc2 + ((size_t)tg * kTCopies + (blockIdx.x & (kTCopies - 1))) * kAccWords;
+}
+
 // A default-mode tile with elements loaded one by one (the last tile of a tensor whose size is
 // not a multiple of 4, or a misaligned tensor): its sums are reduced across the warp at once,
-// fp32 part and fp64 part, and lane 0 stores the tile's kAcc partials.
-__device__ __noinline__ void store_tile_now(double *P, const float (&accf)[kAcc],
-                                            const int (&acce)[kAcc], const double (&accd)[kAcc],
-                                            uint64_t keep) {
+// fp32 part and fp64 part, and lane 0 adds both into the tensor's accumulators.
+__device__ __noinline__ void add_tile_now(const Scalars &sc, int tg, const float (&accf)[kAcc],
+                                          const int (&acce)[kAcc], const double (&accd)[kAcc]) {
     float f[kAcc];
     double d[kAcc];
 #pragma unroll
@@ -1023,8 +1115,14 @@ __device__ __noinline__ void store_tile_now(double *P, const float (&accf)[kAcc]
     warp_sums<kAcc>(d);
     if ((threadIdx.x & 31) == 0) {
 #pragma unroll
-        for (int a = 0; a < kAcc; ++a)
-            st_keep_l2(P + a, __dadd_rn(widen_scaled(f[a], -2 * acce[a]), d[a]), keep);
+        for (int a = 0; a < kAcc; ++a) {
+            acc_add_f32(acc1_of(sc, tg, a), f[a], -2 * acce[a]);
+            acc_add_f64(acc1_of(sc, tg, a), d[a]);
+        }
+        if (sc.mode == kModeStep) {
+            acc_add_f32(gacc_of(sc), f[0], -2 * acce[0]);
+            acc_add_f64(gacc_of(sc), d[0]);
+        }
     }
 }
 
@@ -1036,13 +1134,14 @@ __global__ void __launch_bounds__(Ring1For<PR>::kThreads, 1)
     extern __shared__ __align__(128) unsigned char smem[];
     // In a step that does not read w, the first launch of the pass starts at
     // once.  It can only have been started early by the previous step's pass-2
-    // combine (the update triggers its successor only when that combine
-    // follows), and that combine starts it after its own wait, i.e. once the
-    // previous update has completed: nothing still running then reads the
-    // replicas or the pass-1 partials this kernel writes, and nothing writes
-    // what it loads.  The running combine reads the per-tensor sums the next
-    // combine writes, so this kernel does not complete before it (one wait per
-    // CTA at the end).  Otherwise the whole CTA waits first.
+    // finish (the update triggers its successor only when that finish
+    // follows), and that finish starts it after its own wait, i.e. once the
+    // previous update has completed (and, before it, the pass-1 finish that
+    // re-armed the pass-1 accumulators): nothing still running then reads the
+    // replicas or the pass-1 accumulators this kernel adds into, and nothing
+    // writes what it loads.  The running finish reads the per-tensor sums the
+    // next pass-1 finish writes, so this kernel does not complete before it
+    // (one wait per CTA at the end).  Otherwise the whole CTA waits first.
     grid_launch_dependents();
     const bool early = !RW && !SS && sc.mode == kModeStep && tab.first;
     if (!early) grid_wait();
@@ -1071,9 +1170,10 @@ __global__ void __launch_bounds__(Ring1For<PR>::kThreads, 1)
     const int cw = warp - 1;
     TensorCache tc;
     bool stop = false;
-    const uint64_t keep = policy_evict_last();
+    const bool step_g2 = sc.mode == kModeStep;  // |gbar|^2 also goes into |G|^2
     // The partial sums of a batch of kPend tiles are reduced across the warp together
-    // (reduce-scatter, kRS values with padding) and stored by the lanes that own them.
+    // (reduce-scatter, kRS values with padding) and added into the accumulators by the lanes
+    // that own them.
     constexpr int kRS = 16;
     static_assert(kPend * kAcc <= kRS, "one reduce-scatter per batch");
     for (int jb = cw; !stop; jb += R1::kConsumers * kPend) {
@@ -1083,7 +1183,7 @@ __global__ void __launch_bounds__(Ring1For<PR>::kThreads, 1)
         double pendd[PR ? kRS : 1];
         float pendf[PR ? 1 : kRS];
         unsigned ecode = 0u;
-        int ptile[kPend];
+        int ptensor[kPend];  // global index of each pending tile's tensor, -1: none
 #pragma unroll
         for (int i = 0; i < kRS; ++i) {
             if constexpr (PR) pendd[i] = 0.0;
@@ -1092,7 +1192,7 @@ __global__ void __launch_bounds__(Ring1For<PR>::kThreads, 1)
 #pragma unroll
         for (int p = 0; p < kPend; ++p) {
             const int j = jb + p * R1::kConsumers;
-            ptile[p] = -1;
+            ptensor[p] = -1;
             if (stop) continue;
             // A round-robin tile is located before its wait, a claimed one after.
             int c = j < js ? static_tile(j) : -1;
@@ -1119,31 +1219,38 @@ __global__ void __launch_bounds__(Ring1For<PR>::kThreads, 1)
             __syncwarp();
             if (lane == 0) mbar_arrive(&empty[s]);
             if constexpr (PR) {
-                ptile[p] = tab.c0 + c;
+                ptensor[p] = q.tg;
 #pragma unroll
                 for (int a = 0; a < kAcc; ++a) pendd[p * kAcc + a] = accd[a];
             } else if (tile_tail) {
-                store_tile_now(sc.part1 + (size_t)(tab.c0 + c) * kAcc, accf, acce, accd, keep);
+                add_tile_now(sc, q.tg, accf, acce, accd);
             } else {
-                ptile[p] = tab.c0 + c;
+                ptensor[p] = q.tg;
 #pragma unroll
                 for (int a = 0; a < kAcc; ++a) pendf[p * kAcc + a] = accf[a];
                 ecode |= tcode << (2 * kAcc * p);
             }
         }
         int idx;
-        double v;
-        if constexpr (PR) {
-            v = warp_reduce_scatter<kRS>(pendd, idx);
-        } else {
-            const float f = warp_reduce_scatter<kRS>(pendf, idx);
-            v = widen_scaled(f, -2 * scale_exp((ecode >> (2 * idx)) & 3u));
-        }
+        double vd = 0.0;
+        float vf = 0.f;
+        if constexpr (PR) vd = warp_reduce_scatter<kRS>(pendd, idx);
+        else vf = warp_reduce_scatter<kRS>(pendf, idx);
         // lanes 2i hold value i = p * kAcc + a of the batch
         if ((lane & 1) == 0 && idx < kPend * kAcc) {
             const int p = idx / kAcc, a = idx - p * kAcc;
-            const int t = p == 0 ? ptile[0] : p == 1 ? ptile[1] : p == 2 ? ptile[2] : ptile[3];
-            if (t >= 0) st_keep_l2(sc.part1 + (size_t)t * kAcc + a, v, keep);
+            const int tg = p == 0 ? ptensor[0] : p == 1 ? ptensor[1] : p == 2 ? ptensor[2] : ptensor[3];
+            if (tg >= 0) {
+                unsigned long long *A = acc1_of(sc, tg, a);
+                if constexpr (PR) {
+                    acc_add_f64(A, vd);
+                    if (a == 0 && step_g2) acc_add_f64(gacc_of(sc), vd);
+                } else {
+                    const int k = -2 * scale_exp((ecode >> (2 * idx)) & 3u);
+                    acc_add_f32(A, vf, k);
+                    if (a == 0 && step_g2) acc_add_f32(gacc_of(sc), vf, k);
+                }
+            }
         }
         if (stop) break;
     }
@@ -1151,29 +1258,27 @@ __global__ void __launch_bounds__(Ring1For<PR>::kThreads, 1)
 }
 
 // ----------------------------------------------------------------------------
-// k_combine: per-tensor fixed-order sums of the tile partials
+// k_finish: per-tensor results from the exact accumulators
 // ----------------------------------------------------------------------------
 //
-// One warp per segment of at most kSegTiles tile partials of one tensor (no
-// block barrier; GB300's FP64 pipe sees 15 warp-wide adds per segment).  A
-// tensor of several segments is finished by the warp taking its last segment
-// ticket.  After pass 1 (NA = kAcc) the sums give the tensor's statistics and
-// coefficients; in step mode each tensor then takes a ticket and the warp
-// taking the last one forms |G|^2, Delta and the branch.  After pass 2
-// (NA = 1) the sum is |w|^2 for the statistics.
+// One warp per tensor reads its accumulators (one word per lane), rounds them to fp64
+// (acc_to_double), puts them back to zero for the next call and finishes the tensor: after
+// pass 1 its statistics and coefficient (tensor_done), after pass 2 |w|^2 for the statistics.
+// After pass 1 of a step, one more warp forms |G|^2 from the global accumulator, then Delta
+// (Eq. 5) and the branch of Algorithm 1 (finalize_step).  No warp waits for another.
 
-// Per-tensor results after pass 1, by the whole warp that finished the tensor
-// (its sums in lane 0).  The square roots of |gbar|^2, |g_0|^2 and |w|^2 are
-// taken by lanes 0, 1, 2 in one instruction.
-__device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, double sw,
-                            float old) {
+// Per-tensor results after pass 1, by the whole warp that finished the tensor.  The square
+// roots are taken by lanes 0-2 in one fp64 sequence, and the two divisions likewise by lanes 0
+// and 1: GB300's FP64 pipe is slow, so the lanes share its latency instead of queueing behind it.
+__device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, double sw, float old) {
     const int lane = threadIdx.x & 31;
-    sg = __shfl_sync(kFull, sg, 0);
-    ss = __shfl_sync(kFull, ss, 0);
-    sw = __shfl_sync(kFull, sw, 0);
     const double r = sqrt(lane == 0 ? sg : (lane == 1 ? ss : sw));
     const double ng = __shfl_sync(kFull, r, 0), ns = __shfl_sync(kFull, r, 1),
                  nw = __shfl_sync(kFull, r, 2);
+    // lane 0: UpdateGradScale's ratio |g_s| / (|g_l| + eps); lane 1: |w| / |gbar| (LARS and the
+    // statistics)
+    const double q = (lane == 0 ? ns : nw) / (lane == 0 ? ng + (double)sc.eps : ng);
+    const double q_scale = __shfl_sync(kFull, q, 0), q_w = __shfl_sync(kFull, q, 1);
     if (lane != 0) return;
     double *T = sc.tsum + (size_t)tg * kTsum;
     T[0] = sg;
@@ -1182,7 +1287,7 @@ __device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, dou
     double *row = sc.stats ? sc.stats + (size_t)tg * TULA_STATS_LEN : nullptr;
     if (sc.mode == kModeScale) {
         // UpdateGradScale, g_0 = g_large, small = g_small: min(|g_s| / (|g_l| + eps), s_max)
-        sc.scale[tg] = (float)fmin(ns / (ng + (double)sc.eps), (double)sc.s_max);
+        sc.scale[tg] = (float)fmin(q_scale, (double)sc.s_max);
         return;
     }
     if (sc.mode == kModeStats) {
@@ -1191,7 +1296,7 @@ __device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, dou
         row[TULA_STAT_G0_SQ] = ss;
         row[TULA_STAT_W_NORM] = nw;
         row[TULA_STAT_G_NORM] = ng;
-        row[TULA_STAT_RATIO] = sg > 0.0 ? nw / ng : 0.0;
+        row[TULA_STAT_RATIO] = sg > 0.0 ? q_w : 0.0;
         row[TULA_STAT_COEF] = 0.0;
         row[TULA_STAT_SCALE] = 0.0;
         return;
@@ -1203,7 +1308,7 @@ __device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, dou
     case TULA_RULE_AGS: cand = old; break;
     case TULA_RULE_STATIC: cand = sc.static_s; break;
     case TULA_RULE_LARS:
-        cand = (sw > 0.0 && sg > 0.0) ? (float)((double)sc.lars_trust * (nw / ng)) : 1.0f;
+        cand = (sw > 0.0 && sg > 0.0) ? (float)((double)sc.lars_trust * q_w) : 1.0f;
         break;
     default: cand = 1.0f;
     }
@@ -1211,7 +1316,7 @@ __device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, dou
     float s_after = sc.scale ? old : 0.0f;
     if (sc.refresh && sc.scale) {
         // UpdateGradScale with g_small = replica 0 and g_large = the mean
-        s_after = (float)fmin(ns / (ng + (double)sc.eps), (double)sc.s_max);
+        s_after = (float)fmin(q_scale, (double)sc.s_max);
         sc.scale[tg] = s_after;
     }
     if (row) {
@@ -1222,152 +1327,124 @@ __device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, dou
         if (sc.read_w) {
             row[TULA_STAT_W_SQ] = sw;
             row[TULA_STAT_W_NORM] = nw;
-            row[TULA_STAT_RATIO] = sg > 0.0 ? nw / ng : 0.0;
+            row[TULA_STAT_RATIO] = sg > 0.0 ? q_w : 0.0;
         }
     }
 }
 
-// Eight values added in a fixed pairwise tree (three dependent adds instead of eight).
-__device__ __forceinline__ double sum8(const double (&x)[8]) {
-    return __dadd_rn(__dadd_rn(__dadd_rn(x[0], x[1]), __dadd_rn(x[2], x[3])),
-                     __dadd_rn(__dadd_rn(x[4], x[5]), __dadd_rn(x[6], x[7])));
+// Delta (Eq. 5): this step's |G|^2 against the last step's, +inf at the first step (no previous
+// norm; the step is then unscaled, the sensitive phase).
+__device__ __forceinline__ double variability(double g2, double g2_prev, double steps) {
+    return steps == 0.0 ? (double)INFINITY : fabs((g2 - g2_prev) / g2_prev);
 }
-
-// |G|^2, Delta (Eq. 5) and the branch of Algorithm 1 (one warp, after every
-// segment's |gbar|^2 is in sc.spart1; segments in index order, then a fixed tree).
-__device__ void finalize_step(const Scalars &sc, double g2_prev, double steps) {
-    const double *spart = sc.spart1;
-    const int lane = threadIdx.x & 31;
-    double v[1] = {0.0};
-    for (int g0 = 0; g0 < sc.n_seg1; g0 += 8 * 32) {  // 8 loads in flight per lane
-        double x[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-            const int g = g0 + lane + 32 * u;
-            x[u] = g < sc.n_seg1 ? __ldcg(&spart[(size_t)g * kAcc + 0]) : 0.0;
-        }
-        v[0] = __dadd_rn(v[0], sum8(x));
-    }
-    warp_sums<1>(v);
-    if (lane != 0) return;
-    const double g2 = v[0];
-    // no previous step -> +inf (sensitive)
-    const double dv = steps == 0.0 ? (double)INFINITY : fabs((g2 - g2_prev) / g2_prev);
-    int scaled;
-    if (sc.force == TULA_BRANCH_SCALED) scaled = 1;
-    else if (sc.force == TULA_BRANCH_UNSCALED) scaled = 0;
-    else scaled = dv < (double)sc.delta;  // Algorithm 1: scaled iff Delta < delta
+// The branch of Algorithm 1: scaled iff Delta < delta, unless forced.
+__device__ __forceinline__ int branch_of(const Scalars &sc, double dv) {
+    if (sc.force == TULA_BRANCH_SCALED) return 1;
+    if (sc.force == TULA_BRANCH_UNSCALED) return 0;
+    return dv < (double)sc.delta;
+}
+// The step record from this step's |G|^2 (one lane).
+__device__ void finalize_step(const Scalars &sc, double g2, double g2_prev, double steps) {
+    const double dv = variability(g2, g2_prev, steps);
+    const int scaled = branch_of(sc, dv);
     sc.state[TULA_STATE_G2_PREV] = g2;
     sc.state[TULA_STATE_STEPS] = steps + 1.0;
     sc.state[TULA_STATE_DELTA] = dv;
     sc.state[TULA_STATE_SCALED] = (double)scaled;
     sc.flags[0] = scaled;
-    sc.done[1] = 0u;  // re-arm for the next call
 }
 
-template <int NA>
-__global__ void __launch_bounds__(32 * kCombWarps)
-    k_combine(const __grid_constant__ CombTable tab, const __grid_constant__ Scalars sc) {
-    // Everything that does not come from the kernel before is read ahead of the
-    // wait for it (this kernel is launched early and waits through most of the
-    // previous one): the segment's place in the table and, in a step, the old
-    // gradscale and the step record, which earlier kernels wrote.
+// This lane's word of the sum of R accumulators' Copies copies each (A[r] the first copy of
+// accumulator r): digits and carries added, the flags or-ed.  Every load is issued before the
+// first sum (one round trip); with `rearm`, the copies are put back to zero.
+template <int R, int Copies>
+__device__ __forceinline__ void acc_words(unsigned long long *const (&A)[R], bool rearm,
+                                          unsigned long long (&w)[R]) {
     const int lane = threadIdx.x & 31;
-    const int seg = (int)blockIdx.x * kCombWarps + (int)(threadIdx.x >> 5);
-    const bool active = seg < tab.ns;
-    const int t = active ? tab.seg_t[seg] : 0;
-    const int tg = tab.t0 + t;
-    const int k = seg - tab.sfirst[t];                 // segment within the tensor
-    const int nseg = tab.sfirst[t + 1] - tab.sfirst[t];
-    const long long first = (long long)tab.cfirst[t] + (long long)k * kSegTiles;
-    const int n = min(kSegTiles, tab.ntiles[t] - k * kSegTiles);
-    const bool step = NA == kAcc && sc.mode == kModeStep;
-    const float scale_old = (active && step && sc.scale) ? sc.scale[tg] : 1.0f;
-    const double g2_prev = step ? sc.state[TULA_STATE_G2_PREV] : 0.0;
-    const double steps = step ? sc.state[TULA_STATE_STEPS] : 0.0;
+#pragma unroll
+    for (int r = 0; r < R; ++r) w[r] = 0ull;
+    if (lane >= kAccWords) return;
+    unsigned long long x[R][Copies];
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+#pragma unroll
+        for (int c = 0; c < Copies; ++c) x[r][c] = __ldcg(A[r] + c * kAccWords + lane);
+#pragma unroll
+    for (int r = 0; r < R; ++r)
+#pragma unroll
+        for (int c = 0; c < Copies; ++c) w[r] = lane == kAccFlags ? (w[r] | x[r][c]) : (w[r] + x[r][c]);
+    if (rearm) {
+#pragma unroll
+        for (int r = 0; r < R; ++r)
+#pragma unroll
+            for (int c = 0; c < Copies; ++c) A[r][c * kAccWords + lane] = 0ull;
+    }
+}
+// One accumulator's value (its copies summed), rounded to fp64 by the whole warp.
+template <int Copies>
+__device__ __forceinline__ double acc_read(unsigned long long *A, bool rearm) {
+    unsigned long long *const a[1] = {A};
+    unsigned long long w[1];
+    acc_words<1, Copies>(a, rearm, w);
+    double v[1];
+    acc_to_double<1>(w, v);
+    return v[0];
+}
+
+// |w|^2 of tensor t from pass 2 into its statistics row (lanes 0 and 1 take the two square
+// roots in one instruction).
+__device__ __forceinline__ void w_stats(const Scalars &sc, int t, double sw, double sg) {
+    const int lane = threadIdx.x & 31;
+    const double r = sqrt(lane == 0 ? sw : sg);
+    const double nw = __shfl_sync(kFull, r, 0), ng = __shfl_sync(kFull, r, 1);
+    if (lane == 0) {
+        double *row = sc.stats + (size_t)t * TULA_STATS_LEN;
+        row[TULA_STAT_W_SQ] = sw;
+        row[TULA_STAT_W_NORM] = nw;
+        row[TULA_STAT_RATIO] = sg > 0.0 ? nw / ng : 0.0;
+    }
+}
+
+// NA = kAcc: after pass 1 (the pass-1 norms; in a step also the branch, which the update then
+// reads).  NA = 1: after pass 2 (|w|^2 for the statistics).
+template <int NA>
+__global__ void __launch_bounds__(32 * kFinWarps) k_finish(const __grid_constant__ Scalars sc) {
+    constexpr bool P1 = NA == kAcc;  // pass-1 accumulators
+    const int lane = threadIdx.x & 31;
+    const int t = (int)blockIdx.x * kFinWarps + (int)(threadIdx.x >> 5);
+    const int n = sc.n_total;
+    const bool step = P1 && sc.mode == kModeStep;
+    const bool active = t < n + (step ? 1 : 0);
+    // This kernel is launched early and waits here for the kernel before it; the old gradscale
+    // and the step record are read after the wait, together with the accumulators (no round
+    // trip is added, and no kernel of an earlier call can still be writing them).
     grid_wait();
-    // Inside a step the successor (the update, or the next step's reduction)
-    // may start now; after tula_layer_stats or tula_ags_update_scale it starts
-    // when this kernel has completed (a step's reduction that starts early
-    // overwrites the tile partials this kernel reads).
+    // Inside a step the successor (the update, or the next step's reduction) may start now;
+    // after tula_layer_stats or tula_ags_update_scale it starts when this kernel has completed
+    // (a step's reduction that starts early adds into the accumulators this kernel reads).
     if (sc.mode == kModeStep || NA == 1) grid_launch_dependents();
     if (!active) return;
-    const double *part = NA == kAcc ? sc.part1 : sc.part2;
-    double *spart = NA == kAcc ? sc.spart1 : sc.spart2;
-    unsigned *sctr = NA == kAcc ? sc.sctr1 : sc.sctr2;
-
-    // The segment's tiles: lane i adds tiles i, i + 32, ... in order (8 loads in
-    // flight), then a fixed tree across the warp.
-    double v[NA];
-#pragma unroll
-    for (int a = 0; a < NA; ++a) v[a] = 0.0;
-    int i = lane;
-    for (; i + 7 * 32 < n; i += 8 * 32) {
-        double x[NA][8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u)
-#pragma unroll
-            for (int a = 0; a < NA; ++a) x[a][u] = part[(first + i + 32 * u) * NA + a];
-#pragma unroll
-        for (int a = 0; a < NA; ++a) v[a] = __dadd_rn(v[a], sum8(x[a]));
+    const float scale_old = (t < n && step && sc.scale) ? sc.scale[t] : 1.0f;
+    const double g2_prev = step ? sc.state[TULA_STATE_G2_PREV] : 0.0;
+    const double steps = step ? sc.state[TULA_STATE_STEPS] : 0.0;
+    if (t == n) {  // the record and the branch
+        const double g2 = acc_read<kGCopies>(sc.gacc, true);
+        if (lane == 0) finalize_step(sc, g2, g2_prev, steps);
+        return;
     }
-    for (; i < n; i += 32) {
-#pragma unroll
-        for (int a = 0; a < NA; ++a) v[a] = __dadd_rn(v[a], part[(first + i) * NA + a]);
-    }
-    warp_sums<NA>(v);
-
-    // The branch needs only |G|^2, so it does not wait for the tensors: in a step,
-    // every segment posts its sums and takes a ticket over all segments, and the
-    // warp taking the last one forms |G|^2, Delta and the branch while the
-    // tensors are being finished.  A tensor of several segments is finished by
-    // the warp taking its last segment ticket, which adds the segment sums in
-    // order.
-    const long long sg0 = (long long)tab.s0 + tab.sfirst[t];
-    int last_all = 0, last_seg = 1;
-    if (nseg > 1 || step) {
-        if (lane == 0) {
-#pragma unroll
-            for (int a = 0; a < NA; ++a) spart[(sg0 + k) * NA + a] = v[a];
-            // the tickets release the stores above; the warp taking a last one acquires
-            if (step) last_all = ticket(&sc.done[1]) == (unsigned)(sc.n_seg1 - 1);
-            if (nseg > 1) last_seg = ticket(&sctr[tg]) == (unsigned)(nseg - 1);
-        }
-        last_all = __shfl_sync(kFull, last_all, 0);
-        last_seg = __shfl_sync(kFull, last_seg, 0);
-    }
-    if (last_all) {
-        fence_acq_rel();
-        finalize_step(sc, g2_prev, steps);
-    }
-    if (!last_seg) return;
-    if (nseg > 1) {
-        fence_acq_rel();
-#pragma unroll
-        for (int a = 0; a < NA; ++a) v[a] = 0.0;
-        for (int j = lane; j < nseg; j += 32) {
-#pragma unroll
-            for (int a = 0; a < NA; ++a) v[a] = __dadd_rn(v[a], __ldcg(&spart[(sg0 + j) * NA + a]));
-        }
-        warp_sums<NA>(v);
-        if (lane == 0) sctr[tg] = 0u;  // re-arm
-    }
-
-    // This warp holds tensor tg's sums (lane 0).
+    unsigned long long *A1 = sc.acc1 + (size_t)t * kAcc * kTCopies * kAccWords;
+    unsigned long long *A2 = sc.acc2 + (size_t)t * kTCopies * kAccWords;
     if constexpr (NA == kAcc) {
-        tensor_done(sc, tg, v[0], v[1], v[2], scale_old);
+        unsigned long long *const a[kAcc] = {A1, A1 + kTCopies * kAccWords,
+                                             A1 + 2 * kTCopies * kAccWords};
+        unsigned long long w[kAcc];
+        acc_words<kAcc, kTCopies>(a, true, w);
+        double v[kAcc];
+        acc_to_double<kAcc>(w, v);
+        tensor_done(sc, t, v[0], v[1], v[2], scale_old);
     } else {
-        // lanes 0 and 1 take the two square roots in one instruction
-        const double sw = __shfl_sync(kFull, v[0], 0);
-        const double sg = sc.tsum[(size_t)tg * kTsum + 0];
-        const double r = sqrt(lane == 0 ? sw : sg);
-        const double nw = __shfl_sync(kFull, r, 0), ng = __shfl_sync(kFull, r, 1);
-        if (lane == 0) {
-            double *row = sc.stats + (size_t)tg * TULA_STATS_LEN;
-            row[TULA_STAT_W_SQ] = sw;
-            row[TULA_STAT_W_NORM] = nw;
-            row[TULA_STAT_RATIO] = sg > 0.0 ? nw / ng : 0.0;
-        }
+        const double sw = acc_read<kTCopies>(A2, true);
+        w_stats(sc, t, sw, sc.tsum[(size_t)t * kTsum + 0]);
     }
 }
 
@@ -1415,29 +1492,31 @@ __device__ __noinline__ float w_cols_scaled(uint32_t w_stage, int nv, float f) {
 }
 
 // A tile of the update with elements loaded one by one: its |w|^2 (fp32 part scaled by 2^(2e),
-// fp64 part) reduced across the warp at once and stored by lane 0.
-__device__ __noinline__ void store_w_tile_now(double *P, float aw, int e, double awt) {
+// fp64 part) reduced across the warp at once and added into the accumulator A by lane 0.
+__device__ __noinline__ void add_w_tile_now(unsigned long long *A, float aw, int e, double awt) {
     float f[1] = {aw};
     double d[1] = {awt};
     warp_sums<1>(f);
     warp_sums<1>(d);
-    if ((threadIdx.x & 31) == 0)
-        st_keep_l2(P, __dadd_rn(widen_scaled(f[0], -2 * e), d[0]), policy_evict_last());
+    if ((threadIdx.x & 31) == 0) {
+        acc_add_f32(A, f[0], -2 * e);
+        acc_add_f64(A, d[0]);
+    }
 }
 
 template <bool HM, bool PE, bool SW>
 __global__ void __launch_bounds__(Ring2::kThreads, 1)
     k_update(const __grid_constant__ Table<kNP2> tab, const __grid_constant__ Scalars sc) {
     extern __shared__ __align__(128) unsigned char smem[];
-    // The first launch of the pass follows the pass-1 combine, which starts it
-    // once the reduction kernel has completed (the combine's own wait).  gbar, w
-    // and m are then final, so the producer streams tiles in while the combine
+    // The first launch of the pass follows the pass-1 finish, which starts it
+    // once the reduction kernel has completed (the finish's own wait).  gbar, w
+    // and m are then final, so the producer streams tiles in while the finish
     // still runs; the branch and the coefficients the consumers apply are the
-    // combine's output, so every consumer waits for its completion first.  The
+    // finish's output, so every consumer waits for its completion first.  The
     // whole CTA waits per element (the producer's stream count depends on the
     // branch) and in later launches of the pass (which share the tile counter
     // with the launch before).
-    // Successors may start early only when the pass-2 combine follows (it waits
+    // Successors may start early only when the pass-2 finish follows (it waits
     // for this kernel); the next step's reduction, when it follows directly,
     // must start after this kernel has completed (see k_reduce).
     if (SW) grid_launch_dependents();
@@ -1481,11 +1560,11 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
         // a tile with elements loaded one by one (fp64, rare) is stored at once instead.
         float pend[kPend];
         unsigned ecode = 0u;
-        int ptile[kPend];
+        int ptensor[kPend];  // global index of each pending tile's tensor, -1: none
 #pragma unroll
         for (int p = 0; p < kPend; ++p) {
             const int j = jb + p * Ring2::kConsumers;
-            ptile[p] = -1;
+            ptensor[p] = -1;
             pend[p] = 0.f;
             if (stop) continue;
             int c = j < js ? static_tile(j) : -1;
@@ -1575,9 +1654,9 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
             }
             if (SW) {
                 if (tile_tail) {
-                    store_w_tile_now(sc.part2 + tab.c0 + c, aw, ew, awt);
+                    add_w_tile_now(acc2_of(sc, q.tg), aw, ew, awt);
                 } else {
-                    ptile[p] = tab.c0 + c;
+                    ptensor[p] = q.tg;
                     pend[p] = aw;
                     if (ew) ecode |= scale_code(ew) << (2 * p);
                 }
@@ -1588,11 +1667,10 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
             int idx;
             const float f = warp_reduce_scatter<kPend>(pend, idx);
             if ((lane & 7) == 0) {
-                const int t = idx == 0 ? ptile[0] : idx == 1 ? ptile[1] : idx == 2 ? ptile[2] : ptile[3];
-                if (t >= 0)
-                    st_keep_l2(sc.part2 + t,
-                               widen_scaled(f, -2 * scale_exp((ecode >> (2 * idx)) & 3u)),
-                               policy_evict_last());
+                const int tg = idx == 0 ? ptensor[0] : idx == 1 ? ptensor[1] : idx == 2 ? ptensor[2] : ptensor[3];
+                if (tg >= 0)
+                    acc_add_f32(acc2_of(sc, tg), f,
+                                -2 * scale_exp((ecode >> (2 * idx)) & 3u));
             }
         }
         if (stop) break;
@@ -1674,56 +1752,47 @@ inline int chunk2(bool hm, bool pe) { return Ring2::tile_elems(2 + (hm ? 1 : 0) 
 inline int chunk1_min(int K) { return chunk1(K, true, K == 1); }
 inline int chunk2_min() { return chunk2(true, true); }
 
-inline long long segs_of(long long tiles) { return (tiles + kSegTiles - 1) / kSegTiles; }
-
 struct Plan {
-    long long c1 = 0, c2 = 0, s1 = 0, s2 = 0;  // tiles and combine segments of each pass
+    long long c1 = 0, c2 = 0;  // tiles of each pass (at the smallest tile sizes)
 };
 
-// Workspace layout.  Every counter and flag precedes `part1`, so zeroing
-// [0, part1) clears all of them.
+// Workspace layout.  Every counter, flag and accumulator precedes `tsum`, so zeroing
+// [0, tsum) clears all of them; the error word is the only one no call clears.
 struct WsLayout {
-    size_t done, flags, err, tiles, sctr1, sctr2, part1, part2, spart1, spart2, tsum, cand, total;
+    size_t flags, err, tiles, acc1, gacc, acc2, tsum, cand, total;
 };
 
-WsLayout ws_layout(int n_tensors, const Plan &pl) {
+WsLayout ws_layout(int n_tensors, const Plan &) {
     size_t off = 0;
     auto take = [&](size_t bytes) {
         size_t o = off;
         off = (off + bytes + 255) & ~size_t(255);
         return o;
     };
+    const size_t acc = sizeof(unsigned long long) * kAccWords;
     WsLayout L;
-    L.done = take(sizeof(unsigned) * 4);
     L.flags = take(sizeof(int) * 4);
     L.err = take(sizeof(unsigned) * 4);
     L.tiles = take(sizeof(unsigned) * 4);
-    L.sctr1 = take(sizeof(unsigned) * (size_t)n_tensors);
-    L.sctr2 = take(sizeof(unsigned) * (size_t)n_tensors);
-    L.part1 = take(sizeof(double) * kAcc * (size_t)pl.c1);
-    L.part2 = take(sizeof(double) * (size_t)pl.c2);
-    L.spart1 = take(sizeof(double) * kAcc * (size_t)pl.s1);
-    L.spart2 = take(sizeof(double) * (size_t)pl.s2);
+    L.acc1 = take(acc * kAcc * kTCopies * (size_t)n_tensors);
+    L.gacc = take(acc * kGCopies);
+    L.acc2 = take(acc * kTCopies * (size_t)n_tensors);
     L.tsum = take(sizeof(double) * kTsum * (size_t)n_tensors);
     L.cand = take(sizeof(float) * (size_t)n_tensors);
     L.total = off;
     return L;
 }
 
+// The tile index of either pass must fit an int, which also keeps every accumulator word's
+// carries within its high half (at most two adds below 2^32 per tile).
 bool valid_numels(const int64_t *numels, int n, int K, Plan *pl) {
     if (!numels || n < 1 || K < 1 || K > TULA_MAX_K) return false;
     const int t1 = chunk1_min(K), t2 = chunk2_min();
     Plan p;
-    // One tensor's tile partials must fit one combine table (see CombTable).
-    const long long max_tiles = (long long)CombTable::kMaxS * kSegTiles;
     for (int i = 0; i < n; ++i) {
         if (numels[i] < 0) return false;
-        const long long a = tiles_of(numels[i], t1), b = tiles_of(numels[i], t2);
-        if (a > max_tiles || b > max_tiles) return false;
-        p.c1 += a;
-        p.c2 += b;
-        p.s1 += segs_of(a);
-        p.s2 += segs_of(b);
+        p.c1 += tiles_of(numels[i], t1);
+        p.c2 += tiles_of(numels[i], t2);
         if (p.c1 >= (1LL << 31) || p.c2 >= (1LL << 31)) return false;
     }
     *pl = p;
@@ -1844,44 +1913,12 @@ int launch_streaming(Kernel kernel, int n, const int64_t *numels, int chunk, int
     return TULA_OK;
 }
 
-// k_combine over all tensors (tiles of `chunk` elements), NA sums per tile.
+// k_finish over all tensors: NA accumulators per tensor (+ the branch after pass 1 of a step).
 template <int NA>
-int launch_combine(int n, const int64_t *numels, int chunk, const Scalars &sc_in, cudaStream_t s) {
-    std::unique_ptr<CombTable> tab(new CombTable);
-    Scalars sc = sc_in;
-    long long segs_total = 0;  // the branch's ticket runs over every segment of every launch
-    for (int p = 0; p < n; ++p) segs_total += segs_of(tiles_of(numels[p], chunk));
-    sc.n_seg1 = (int)segs_total;
-    long long c_global = 0, s_global = 0;
-    int p = 0;
-    while (p < n) {
-        std::memset(tab.get(), 0, sizeof(CombTable));
-        tab->t0 = p;
-        tab->s0 = (int)s_global;
-        int cnt = 0, ns = 0;
-        while (p < n && cnt < CombTable::kMaxT) {
-            const long long c = tiles_of(numels[p], chunk);
-            const int segs = (int)segs_of(c);
-            if (ns + segs > CombTable::kMaxS) break;  // next launch
-            tab->cfirst[cnt] = (int)c_global;
-            tab->ntiles[cnt] = (int)c;
-            tab->sfirst[cnt] = ns;
-            for (int k = 0; k < segs; ++k) tab->seg_t[ns + k] = (unsigned short)cnt;
-            ns += segs;
-            c_global += c;
-            ++cnt;
-            ++p;
-        }
-        if (cnt == 0) return TULA_ERR_ARG;  // excluded up front by valid_numels
-        tab->n = cnt;
-        tab->ns = ns;
-        tab->sfirst[cnt] = ns;
-        s_global += ns;
-        const int grid = (ns + kCombWarps - 1) / kCombWarps;
-        const int rc = launch_pdl(k_combine<NA>, grid, 32 * kCombWarps, 0, s, *tab, sc);
-        if (rc) return rc;
-    }
-    return TULA_OK;
+int launch_finish(int n, const Scalars &sc, cudaStream_t s) {
+    const bool record = NA == kAcc && sc.mode == kModeStep;  // + the branch's warp
+    const int warps = n + (record ? 1 : 0);
+    return launch_pdl(k_finish<NA>, (warps + kFinWarps - 1) / kFinWarps, 32 * kFinWarps, 0, s, sc);
 }
 
 Scalars make_scalars(const tula_ags_hparams *hp, int K, int n, void *ws, const WsLayout &L,
@@ -1909,16 +1946,12 @@ Scalars make_scalars(const tula_ags_hparams *hp, int K, int n, void *ws, const W
         sc.stats = hp->layer_stats;
     }
     char *b = static_cast<char *>(ws);
-    sc.done = reinterpret_cast<unsigned *>(b + L.done);
     sc.flags = reinterpret_cast<int *>(b + L.flags);
     sc.err = reinterpret_cast<unsigned *>(b + L.err);
     sc.tiles = reinterpret_cast<unsigned *>(b + L.tiles);
-    sc.sctr1 = reinterpret_cast<unsigned *>(b + L.sctr1);
-    sc.sctr2 = reinterpret_cast<unsigned *>(b + L.sctr2);
-    sc.part1 = reinterpret_cast<double *>(b + L.part1);
-    sc.part2 = reinterpret_cast<double *>(b + L.part2);
-    sc.spart1 = reinterpret_cast<double *>(b + L.spart1);
-    sc.spart2 = reinterpret_cast<double *>(b + L.spart2);
+    sc.acc1 = reinterpret_cast<unsigned long long *>(b + L.acc1);
+    sc.gacc = reinterpret_cast<unsigned long long *>(b + L.gacc);
+    sc.acc2 = reinterpret_cast<unsigned long long *>(b + L.acc2);
     sc.tsum = reinterpret_cast<double *>(b + L.tsum);
     sc.cand = reinterpret_cast<float *>(b + L.cand);
     return sc;
@@ -1928,7 +1961,7 @@ void record(void *ev, cudaStream_t s) {
     if (ev) cudaEventRecord(static_cast<cudaEvent_t>(ev), s);
 }
 
-// Pass 1 (+ its combine) dispatched over the compile-time replica count.
+// Pass 1 (+ its finish) dispatched over the compile-time replica count.
 template <int KT, bool WM, bool RW, bool SS, bool PR, typename Fill>
 int run_reduce_k(int K, int n, const int64_t *numels, const Scalars &sc, int grid, cudaStream_t s,
                  Fill fill, void *mid_event) {
@@ -1938,7 +1971,7 @@ int run_reduce_k(int K, int n, const int64_t *numels, const Scalars &sc, int gri
                                           grid, s, fill);
     if (rc) return rc;
     record(mid_event, s);
-    return launch_combine<kAcc>(n, numels, chunk, sc, s);
+    return launch_finish<kAcc>(n, sc, s);
 }
 
 template <bool WM, bool RW, bool SS, bool PR, typename Fill>
@@ -2153,7 +2186,7 @@ int run_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mo
 #undef TULA_UPD
     if (rc) return rc;
     record(hp->trace_events[3], s);
-    if (sw) rc = launch_combine<1>(n, numels, c2, sc, s);
+    if (sw) rc = launch_finish<1>(n, sc, s);
     if (rc) return rc;
     record(hp->trace_events[4], s);
     return TULA_OK;
@@ -2322,14 +2355,14 @@ extern "C" int tula_ags_step_static_scratch(float *const *param_ptrs, float *con
     void *scratch = nullptr;
     rc = static_scratch_address(&scratch);
     if (rc) return rc;
-    // The array keeps the last call's contents: zero the tickets, the branch flag and the tile
-    // counters (they precede the partial sums) before this call's kernels.  The error word
-    // between them is left alone, so that a wait that ran out stays reported until
+    // The array keeps the last call's contents: zero the branch flag, the tile counters and the
+    // accumulators (they precede the per-tensor sums) before this call's kernels.  The error
+    // word between them is left alone, so that a wait that ran out stays reported until
     // tula_ags_static_scratch_error reads it.
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     char *b = static_cast<char *>(scratch);
     cudaError_t e = cudaMemsetAsync(b, 0, L.err, s);
-    if (e == cudaSuccess) e = cudaMemsetAsync(b + L.tiles, 0, L.part1 - L.tiles, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(b + L.tiles, 0, L.tsum - L.tiles, s);
     if (e != cudaSuccess) {
         g_last_cuda = (int)e;
         return TULA_ERR_CUDA;

@@ -241,11 +241,11 @@ def test_steps_replayed_from_a_cuda_graph():
     assert steps[0].state[1].item() == 5.0  # five steps taken: the refresh step and four more
 
 
-def test_largest_tensor_the_library_takes():
-    """One tensor at the per-tensor limit (K = 2: 1,694,208 tiles of 1536 elements, 2.6e9
-    elements, past 2^31), constant per role so that every element has the same closed-form
-    result, which the oracle gives on a few elements: sampled elements around 2^31 and at both
-    ends, the extremes over the whole tensor, and |G|^2 = n |gbar|^2."""
+def test_a_tensor_past_2_31_elements():
+    """One tensor of 2.6e9 elements (K = 2; element indices past 2^31), constant per role so
+    that every element has the same closed-form result, which the oracle gives on a few
+    elements: sampled elements around 2^31 and at both ends, the extremes over the whole
+    tensor, and |G|^2 = n |gbar|^2."""
     K = 2
     n = 1_694_208 * min(T.tula_ags_chunk_elems(1, K + 1), T.tula_ags_chunk_elems(2, 4))
     assert n > 2 ** 31
@@ -518,3 +518,55 @@ def test_default_steps_misaligned_over_the_whole_float_range(K):
         pair.step(1, 1.0)
         pair.step(1, 1.0)
         assert pair.flags == [0, 1]
+
+
+@pytest.mark.parametrize("K", [1, 8])
+def test_norms_are_exact_sums_on_integer_data(K):
+    """With small integers in every replica and weight, every square and every fp32 tile sum is
+    exact, so the exact accumulation across tiles must give the oracle's norms bit for bit (the
+    oracle's compensated fp64 sums are exact here too), and |G|^2 must be the exact sum of the
+    per-tensor |gbar|^2, for any grid size."""
+    ps = _ragged_pset(extra=(3_000_001,), K=K)
+    wl = W.workload("stress_k4", seed=131 + K, zero_patterns=False)
+    buf = W.allocate(wl, "cuda", K=K, pset=ps)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(131 + K)
+    for f in [buf.w_flat] + buf.g_flats:
+        f.copy_(torch.randint(-7, 8, f.shape, generator=gen, device="cuda").float())
+    ref = O.layer_stats(W.to_numpy(buf.w), [W.to_numpy(buf.g[k]) for k in range(K)])
+    cols = (T.TULA_STAT_W_SQ, T.TULA_STAT_G_SQ, T.TULA_STAT_G0_SQ)
+    for col in cols:
+        assert np.all(ref[:, col] == np.round(ref[:, col] * 64) / 64)  # exact, as claimed
+    g2 = float(np.sum(ref[:, T.TULA_STAT_G_SQ]))  # exact: every term a multiple of 1/64
+    stats = torch.zeros(buf.pset.n_tensors, 8, dtype=torch.float64, device="cuda")
+    T.tula_layer_stats(buf.w, buf.g, stats, T.new_workspace(buf.numels, K))
+    torch.cuda.synchronize()
+    for col in cols:
+        assert np.array_equal(stats.cpu().numpy()[:, col], ref[:, col]), ("layer_stats", col)
+    snap = _inputs_snapshot(buf)
+    for grid in (0, 1, 13, 333):
+        _restore(buf, snap)
+        st = T.AGSOptimizerStep(buf.w, buf.g, buf.m, grid_ctas=grid)
+        st.step(0.1, 0.9, 0.0)
+        torch.cuda.synchronize()
+        got = st.stats.cpu().numpy()
+        for col in cols:
+            assert np.array_equal(got[:, col], ref[:, col]), (grid, col)
+        assert st.state[0].item() == g2, grid
+
+
+@pytest.mark.parametrize("n", [1, 3, 4, 5, 8, 9])
+@pytest.mark.parametrize("rule", [T.TULA_RULE_AGS, T.TULA_RULE_LARS])
+def test_tensor_counts_around_a_finish_block(n, rule):
+    """The finish kernel runs one warp per tensor, four per block, plus one warp for the step
+    record: tensor counts that fill whole blocks, and those that do not, both get their record
+    (|G|^2, Delta, branch) and every tensor's statistics, in the step that takes the branch in
+    the update (AGS) and in the one with a finish between the passes (LARS)."""
+    ps = W.ParamSet("count")
+    for i in range(n):
+        ps.add((1000 + 517 * i,), W.KIND_NORMAL)
+    wl = W.workload("stress_k4", seed=141 + n, factor_range=(0.1, 10.0), zero_patterns=False)
+    pair = Pair(wl, K=2, pset=ps, rule=rule, lars_trust=0.01)
+    for seed_step, mult in ((1, 1.0), (1, 1.0), (1, 2.0)):
+        pair.step(seed_step, mult)
+    assert pair.flags == [0, 1, 0]

@@ -28,13 +28,15 @@ def test_rejects_tensor_lists_beyond_the_static_scratch():
     CUDA call (the pointers below are never dereferenced)."""
     B.build()
     lib = T.lib()
-    numels = [1 << 30] * 64  # 2^36 elements: ~0.9 GB of tile partials, far beyond 16 MiB
+    n = 5500  # about 3.1 KB of scratch per tensor: 17 MB, beyond 16 MiB
+    numels = [5] * n
     assert T.tula_ags_workspace_size(numels, 1) > T.TULA_STATIC_SCRATCH_BYTES
+    assert T.tula_ags_workspace_size(numels[:5300], 1) <= T.TULA_STATIC_SCRATCH_BYTES
     P = ctypes.c_void_p
-    ptrs = (P * 64)(*[0x100000 * (i + 1) for i in range(64)])
+    ptrs = (P * n)(*[0x100000 * (i + 1) for i in range(n)])
     hp = T.tula_ags_default_hparams(1)
     hp.scale, hp.state = 0x200000, 0x300000
-    rc = lib.tula_ags_step_static_scratch(ptrs, ptrs, ptrs, (ctypes.c_int64 * 64)(*numels), 64,
+    rc = lib.tula_ags_step_static_scratch(ptrs, ptrs, ptrs, (ctypes.c_int64 * n)(*numels), n,
                                           0.1, 0.9, 0.0, ctypes.byref(hp), None)
     assert rc == T.TULA_ERR_SCRATCH_LIMIT
     assert "static scratch" in T.tula_ags_error_string(rc)
