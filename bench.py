@@ -8,10 +8,13 @@ update pass over a whole parameter set) on GB300.
 Prints ONE JSON line.  `value` is parameters updated per second over the whole
 job, device-resident inputs; `e2e` is the same metric through the C ABI with
 the replica gradients copied in from pinned host memory and the step record and
-per-layer statistics copied back inside the timed region.  Under torchrun every
-rank runs its own replica step on its own GPU (no collective on the data path:
-one optimizer step has nothing to exchange once the K replicas are local), and
-the time is the max over ranks.
+per-layer statistics copied back inside the timed region.  `secondary` holds the
+same step timed on the VGG-16 parameter set (the other set the roofline target
+names), and `cpu_baseline` the CPU oracle on all host cores, with its
+single-threaded figure beside it.  Under torchrun every rank runs its own
+replica step on its own GPU (no collective on the data path: one optimizer step
+has nothing to exchange once the K replicas are local), and the time is the max
+over ranks.
 """
 from __future__ import annotations
 
@@ -47,6 +50,13 @@ def _args():
                     help="untimed load before the timed steps, so clock samples see load")
     ap.add_argument("--cpu-sample-s", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-secondary", dest="secondary", action="store_false",
+                    help="skip the second parameter set (VGG-16) timed after the headline one")
+    ap.add_argument("--granularity", default="tensor", choices=["tensor", "element"],
+                    help="gradscale per tensor (default) or per element (Algorithm 1's line "
+                         "read literally; the update then reads a scale per parameter)")
+    ap.add_argument("--no-momentum", dest="momentum", action="store_false",
+                    help="steps without a momentum buffer (w -= lr * d)")
     ap.add_argument("--step-kind", default="ags", choices=list(STEP_KINDS),
                     help="ags: Algorithm 1 steps (the gradscale refreshed once, in warm-up); "
                          "refresh: every step also refreshes the gradscale (UpdateGradScale fused "
@@ -85,7 +95,8 @@ def job_throughput(params_per_rank: int, steps: int, world_size: int, t_max_ms: 
 
 LARS_TRUST = 1e-3  # trust coefficient of the LARS steps timed here
 # step kind -> (reads w in pass 1, refreshes the gradscale every step)
-STEP_KINDS = {"ags": (False, False), "refresh": (False, True), "lars": (True, False)}
+STEP_KINDS = {"ags": (False, False), "refresh": (False, True), "lars": (True, False),
+              "update-scale": (False, False)}
 
 
 def pass1_bytes_per_param(K: int, read_w: bool = False) -> int:
@@ -93,21 +104,31 @@ def pass1_bytes_per_param(K: int, read_w: bool = False) -> int:
     return 4 * K + (4 if K > 1 else 0) + (4 if read_w else 0)
 
 
-def pass2_bytes_per_param(with_momentum=True) -> int:
-    """Update pass: read gbar, w, m; write w, m."""
-    return 20 if with_momentum else 12
+def pass2_bytes_per_param(with_momentum=True, per_element=False) -> int:
+    """Update pass: read gbar, w, m; write w, m (no momentum buffer: read gbar, w; write w).  A
+    per-element gradscale is read too (in a scaled step)."""
+    return (20 if with_momentum else 12) + (4 if per_element else 0)
 
 
-def step_design_bytes_per_param(K: int, read_w: bool = False) -> int:
+def step_design_bytes_per_param(K: int, read_w: bool = False, with_momentum=True,
+                                per_element=False) -> int:
     """What the two passes move as built: pass 1 plus pass 2 (the mean is written over
     replica 0 and read back by the update, as an in-place all-reduce would leave it)."""
-    return pass1_bytes_per_param(K, read_w) + pass2_bytes_per_param()
+    return pass1_bytes_per_param(K, read_w) + pass2_bytes_per_param(with_momentum, per_element)
 
 
-def step_min_bytes_per_param(K: int, read_w: bool = False) -> int:
+def step_min_bytes_per_param(K: int, read_w: bool = False, with_momentum=True,
+                             per_element=False) -> int:
     """Algorithmic minimum of one step: read K replicas, w, m; write w, m (LARS: w is read
-    once more, since its norm sets the coefficient before the update)."""
-    return 4 * K + 16 + (4 if read_w else 0)
+    once more, since its norm sets the coefficient before the update; no momentum buffer: 8
+    bytes less; a per-element gradscale: 4 more)."""
+    return (4 * K + 16 + (4 if read_w else 0) - (0 if with_momentum else 8)
+            + (4 if per_element else 0))
+
+
+def scale_elem_bytes_per_param() -> int:
+    """UpdateGradScale element-wise: read g_small and g_large, write the scale."""
+    return 12
 
 
 # ---------------------------------------------------------------------------
@@ -236,7 +257,14 @@ def _host_inputs(wl, frac=1.0):
     return pset, w, m, g
 
 
-def _oracle_steps(wl, w, m, g, steps, kind="ags"):
+def host_cores() -> int:
+    """Threads the all-cores oracle runs on: the host's CPU count (bounded by what the oracle's
+    OpenMP build can use)."""
+    import oracle as O
+    return max(1, min(os.cpu_count() or 1, O.max_threads()))
+
+
+def _oracle_steps(wl, w, m, g, steps, kind="ags", threads=None):
     import numpy as np
 
     import oracle as O
@@ -247,21 +275,33 @@ def _oracle_steps(wl, w, m, g, steps, kind="ags"):
     state = O.new_state()
     t0 = time.perf_counter()
     for _ in range(steps):
-        O.ags_step(w, m, g, wl.lr, wl.momentum, wl.weight_decay, hp, scale=scale, state=state)
+        O.ags_step(w, m, g, wl.lr, wl.momentum, wl.weight_decay, hp, scale=scale, state=state,
+                   threads=threads)
     return time.perf_counter() - t0
 
 
-def cpu_baseline(wl, budget_s, kind="ags"):
-    """The oracle as it stands (single-threaded C) on the host: a bounded number of
-    full optimizer steps over the same parameter set."""
-    pset, w, m, g = _host_inputs(wl)
-    t1 = _oracle_steps(wl, w, m, g, 1, kind)
+def _timed_oracle(wl, pset, w, m, g, budget_s, kind, threads):
+    t1 = _oracle_steps(wl, w, m, g, 1, kind, threads)
     steps = max(1, min(50, int(budget_s / max(t1, 1e-6))))
-    t = _oracle_steps(wl, w, m, g, steps, kind)
-    return {"value": pset.n_params * steps / t, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{steps} full steps of the {wl.name} parameter set "
-                      f"({pset.n_params} params, {pset.n_tensors} tensors, K={wl.K}) on the host, "
-                      f"single-threaded C oracle"}
+    t = _oracle_steps(wl, w, m, g, steps, kind, threads)
+    return pset.n_params * steps / t, steps
+
+
+def cpu_baseline(wl, budget_s, kind="ags"):
+    """The oracle as it stands on the host: a bounded number of full optimizer steps over the
+    same parameter set, on all host cores (its per-tensor parts in parallel, the combine in
+    tensor order; bitwise the single-threaded result) and on one core."""
+    pset, w, m, g = _host_inputs(wl)
+    cores = host_cores()
+    v_all, s_all = _timed_oracle(wl, pset, w, m, g, budget_s / 2, kind, cores)
+    v_one, s_one = _timed_oracle(wl, pset, w, m, g, budget_s / 2, kind, None)
+    what = (f"full steps of the {wl.name} parameter set ({pset.n_params} params, "
+            f"{pset.n_tensors} tensors, K={wl.K}) on the host, C oracle")
+    return {"value": v_all, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{s_all} {what}, per-tensor parts on {cores} threads",
+            "host_cpu_count": os.cpu_count(),
+            "single_thread": {"value": v_one, "unit": UNIT, "cores": 1,
+                              "sample": f"{s_one} {what}, one thread"}}
 
 
 def run_reference(args, wl):
@@ -270,20 +310,23 @@ def run_reference(args, wl):
         return
     pset_full = wl.pset
     kind = args.step_kind
+    if kind == "update-scale":
+        raise SystemExit("--impl reference times optimizer steps, not --step-kind update-scale")
     if STEP_KINDS[kind][1] and wl.K == 1:
         raise SystemExit("--step-kind refresh needs K > 1 (g_small is replica 0)")
     _, w, m, g = _host_inputs(wl)
-    t1 = _oracle_steps(wl, w, m, g, 1, kind)
+    cores = host_cores()
+    t1 = _oracle_steps(wl, w, m, g, 1, kind, cores)
     total = args.steps + args.warmup
     frac = min(1.0, 120.0 / max(1e-9, total * t1))
     if frac < 1.0:
         pset, w, m, g = _host_inputs(wl, frac)
     else:
         pset = pset_full
-    _oracle_steps(wl, w, m, g, args.warmup, kind)
-    t = _oracle_steps(wl, w, m, g, args.steps, kind)
+    _oracle_steps(wl, w, m, g, args.warmup, kind, cores)
+    t = _oracle_steps(wl, w, m, g, args.steps, kind, cores)
     value = pset.n_params * args.steps / t
-    sample = (f"each step: the single-threaded C oracle over "
+    sample = (f"each step: the C oracle, per-tensor parts on {cores} threads, over "
               f"{'all' if frac >= 1.0 else 'the first'} {pset.n_tensors} tensors "
               f"({pset.n_params} of {pset_full.n_params} params) of the {wl.name} set, K={wl.K}")
     line = {
@@ -291,8 +334,8 @@ def run_reference(args, wl):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * t / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic", "config": _config(wl, pset_full, kind),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                         "sample": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": sample, "host_cpu_count": os.cpu_count()},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -300,15 +343,22 @@ def run_reference(args, wl):
 
 STEP_KIND_TEXT = {
     "ags": "Algorithm 1 step (AGS rule, per-tensor gradscale)",
+    "update-scale": "UpdateGradScale of Algorithm 1 alone, element-wise (g_small = replica 1, "
+                    "g_large = replica 0): not a step",
     "refresh": "Algorithm 1 step that also refreshes the gradscale (UpdateGradScale, g_small = "
                "replica 0)",
     "lars": "LARS rule step (coefficient 0.001 |w| / |gbar|)",
 }
 
 
-def _config(wl, pset, kind="ags"):
+def _config(wl, pset, kind="ags", per_elem=False, momentum=True):
+    step = STEP_KIND_TEXT[kind]
+    if per_elem:
+        step += "; gradscale per element"
+    if not momentum:
+        step += "; no momentum buffer"
     return {"workload": f"{wl.name} parameter set, K={wl.K} replica gradient buffers",
-            "step": STEP_KIND_TEXT[kind],
+            "step": step,
             "params": pset.n_params, "tensors": pset.n_tensors, "K": wl.K,
             "global_batch": None, "seq_len": None, "parallelism": "replicas only (1 step per GPU)",
             "l2": "inputs larger than L2 (no flush): "
@@ -319,6 +369,75 @@ def _config(wl, pset, kind="ags"):
 # ---------------------------------------------------------------------------
 # GPU timing
 # ---------------------------------------------------------------------------
+
+SECONDARY = "vgg16"  # the other parameter set the >= 80 % roofline target names
+
+
+def secondary_record(name, args, kind, stream, peak):
+    """The step on a second parameter set, timed the same way as the headline (steps back to
+    back on one stream, CUDA events; then the same steps again with events at the kernel
+    boundaries for the per-kernel fractions).  Inputs are device-resident; its tensors are
+    freed before returning."""
+    import torch
+
+    from paper_2603_18112_gb300 import tula_ags as T
+    from paper_2603_18112_gb300 import workloads as W
+    wl = W.workload(name)
+    read_w, refresh = STEP_KINDS[kind]
+    if refresh and wl.K == 1:
+        return None
+    N, K = wl.pset.n_params, wl.K
+    buf = W.allocate(wl, "cuda")
+    W.fill_state(buf, wl)
+    W.fill_grads(buf, wl, step=1)
+    torch.cuda.synchronize()
+    step = T.AGSOptimizerStep(buf.w, buf.g, buf.m, s_max=wl.smax,
+                              rule=T.TULA_RULE_LARS if kind == "lars" else T.TULA_RULE_AGS,
+                              lars_trust=LARS_TRUST)
+    steps = max(1, min(args.steps, 100))
+    with torch.cuda.stream(stream):
+        for i in range(max(3, args.warmup)):
+            step.step(wl.lr, wl.momentum, wl.weight_decay,
+                      refresh_scale=refresh or (kind == "ags" and i == 0 and K > 1), stream=stream)
+    stream.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(steps):
+            step.step(wl.lr, wl.momentum, wl.weight_decay, refresh_scale=refresh, stream=stream)
+        t1.record(stream)
+    stream.synchronize()
+    ms = t0.elapsed_time(t1) / steps
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(steps)]
+    with torch.cuda.stream(stream):
+        for e5 in evs:  # recorded once by torch, so that it times them
+            for e in e5:
+                e.record(stream)
+        for e5 in evs:
+            step.set_trace_events(e5)
+            step.step(wl.lr, wl.momentum, wl.weight_decay, refresh_scale=refresh, stream=stream)
+    step.set_trace_events(None)
+    torch.cuda.synchronize()
+    red = statistics.fmean(e[0].elapsed_time(e[1]) for e in evs)
+    upd = statistics.fmean(e[2].elapsed_time(e[3]) for e in evs)
+    p1 = pass1_bytes_per_param(K, read_w) * N
+    p2 = pass2_bytes_per_param() * N
+    step_gbs = step_min_bytes_per_param(K, read_w) * N / (ms / 1e3) / 1e9
+    out = {"workload": f"{name} parameter set, K={K} replica gradient buffers",
+           "params": N, "tensors": wl.pset.n_tensors, "steps": steps, "ms_per_step": ms,
+           "value": N / (ms / 1e3), "unit": UNIT,
+           "k_reduce": {"ms_per_launch": red, "bytes_per_launch": p1,
+                        "frac": p1 / (red / 1e3) / 1e9 / peak},
+           "k_update": {"ms_per_launch": upd, "bytes_per_launch": p2,
+                        "frac": p2 / (upd / 1e3) / 1e9 / peak},
+           "step_hbm": {"algorithmic_bytes_per_param": step_min_bytes_per_param(K, read_w),
+                        "achieved_gbs": step_gbs, "frac": step_gbs / peak,
+                        "frac_of_8tbs": step_gbs / 8000.0},
+           "l2": "inputs larger than L2 (no flush)"}
+    del step, buf
+    torch.cuda.empty_cache()
+    return out
+
 
 def run_ours(args, wl):
     import torch
@@ -343,20 +462,30 @@ def run_ours(args, wl):
     read_w, refresh = STEP_KINDS[kind]
     if refresh and K == 1:
         raise SystemExit("--step-kind refresh needs K > 1 (g_small is replica 0)")
-    buf = W.allocate(wl, "cuda")
+    per_elem = args.granularity == "element"
+    mu = wl.momentum if args.momentum else 0.0
+    buf = W.allocate(wl, "cuda", with_momentum=args.momentum)
     W.fill_state(buf, wl)
     W.fill_grads(buf, wl, step=1)
     stream = torch.cuda.Stream()
+    scale_elem = None
+    if per_elem:  # a per-element gradscale in [0.5, 2]
+        gen = torch.Generator(device="cuda")
+        gen.manual_seed(wl.seed * 7919 + 5)
+        scale_elem = [torch.rand(t.shape, generator=gen, device="cuda") * 1.5 + 0.5 for t in buf.w]
     torch.cuda.synchronize()
     # LARS with a trust coefficient of 1 moves w by about |w| each step: on one gradient reused
     # for thousands of steps the weights overflow within ~120 steps, and every tile then takes
     # the exact-fp64 fallback of the precise norms.  0.001 keeps them bounded.
-    step = T.AGSOptimizerStep(buf.w, buf.g, buf.m, s_max=wl.smax,
+    step = T.AGSOptimizerStep(buf.w, buf.g, buf.m if args.momentum else None, s_max=wl.smax,
                               rule=T.TULA_RULE_LARS if kind == "lars" else T.TULA_RULE_AGS,
-                              lars_trust=LARS_TRUST)
+                              lars_trust=LARS_TRUST,
+                              granularity=(T.TULA_SCALE_PER_ELEMENT if per_elem
+                                           else T.TULA_SCALE_PER_TENSOR),
+                              scale_elem=scale_elem)
 
     def one_step():
-        step.step(wl.lr, wl.momentum, wl.weight_decay, refresh_scale=refresh, stream=stream)
+        step.step(wl.lr, mu, wl.weight_decay, refresh_scale=refresh, stream=stream)
 
     def barrier():
         if ws > 1:
@@ -365,8 +494,8 @@ def run_ours(args, wl):
     with torch.cuda.stream(stream):
         for i in range(args.warmup):
             # the first warm-up step refreshes the gradscale (UpdateGradScale needs K > 1)
-            step.step(wl.lr, wl.momentum, wl.weight_decay,
-                      refresh_scale=refresh or (kind == "ags" and i == 0 and K > 1),
+            step.step(wl.lr, mu, wl.weight_decay,
+                      refresh_scale=refresh or (kind == "ags" and i == 0 and K > 1 and not per_elem),
                       stream=stream)
     stream.synchronize()
 
@@ -402,6 +531,20 @@ def run_ours(args, wl):
     torch.cuda.synchronize()
     barrier()
     launches = T.tula_ags_launch_count() - launches0
+    # Host time per call: 50 steps issued after a synchronize, timed on the host up to the
+    # return of the last call (the launch queue holds them all, so the host never waits on
+    # the GPU unless it is the faster side).
+    torch.cuda.synchronize()
+    h0 = time.perf_counter()
+    with torch.cuda.stream(stream):
+        for _ in range(50):
+            one_step()
+    host_us = (time.perf_counter() - h0) / 50 * 1e6
+    torch.cuda.synchronize()
+    peak, peak_kind = _peaks()
+    secondary = (secondary_record(SECONDARY, args, kind, stream, peak)
+                 if args.secondary and wl.name != SECONDARY and not per_elem and args.momentum
+                 else None)
     clocks = sampler.stop()
     elapsed_ms = t_start.elapsed_time(t_end)
     # Per-pass times: the same steps again, with the library recording events at the pass
@@ -453,14 +596,15 @@ def run_ours(args, wl):
         dist.destroy_process_group()
         return
 
-    peak, peak_kind = _peaks()
     p1_avg_ms = statistics.fmean(t_red)
     p2_avg_ms = statistics.fmean(t_upd)
     p1_bytes = pass1_bytes_per_param(K, read_w) * N
-    p2_bytes = pass2_bytes_per_param() * N
+    p2_bytes = pass2_bytes_per_param(args.momentum, per_elem) * N
     achieved = p1_bytes / (p1_avg_ms / 1e3) / 1e9
     ms_per_step = t_max_ms / args.steps
-    step_gbs = step_min_bytes_per_param(K, read_w) * N / (ms_per_step / 1e3) / 1e9
+    smin = step_min_bytes_per_param(K, read_w, args.momentum, per_elem)
+    sdes = step_design_bytes_per_param(K, read_w, args.momentum, per_elem)
+    step_gbs = smin * N / (ms_per_step / 1e3) / 1e9
     red_name = "k_reduce" if kind == "ags" else f"k_reduce_{kind}"
     traffic = _ncu_traffic(red_name, wl.name, N)
     line = {
@@ -468,7 +612,7 @@ def run_ours(args, wl):
         "n_gpus": ws, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
         "steps_per_s": 1e3 / ms_per_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": _config(wl, pset, kind),
+        "config": _config(wl, pset, kind, per_elem, args.momentum),
         "roofline": {"bound": "hbm",
                      "kernel": "k_reduce (replica mean + tile norms"
                                + (")" if kind == "ags" else ", precise norms)"),
@@ -482,13 +626,14 @@ def run_ours(args, wl):
                         "frac": p2_bytes / (p2_avg_ms / 1e3) / 1e9 / peak},
         "combine_ms": {"after_reduce": statistics.fmean(t_cmb1),
                        "after_update": statistics.fmean(t_cmb2)},
-        "step_hbm": {"algorithmic_bytes_per_param": step_min_bytes_per_param(K, read_w),
+        "step_hbm": {"algorithmic_bytes_per_param": smin,
                      "achieved_gbs": step_gbs, "frac": step_gbs / peak,
                      "frac_of_8tbs": step_gbs / 8000.0,
-                     "design_bytes_per_param": step_design_bytes_per_param(K, read_w),
-                     "design_gbs": step_design_bytes_per_param(K, read_w) * N
-                     / (ms_per_step / 1e3) / 1e9},
+                     "design_bytes_per_param": sdes,
+                     "design_gbs": sdes * N / (ms_per_step / 1e3) / 1e9},
         "e2e": e2e,
+        "host_us_per_call": host_us,
+        "secondary": [secondary] if secondary else [],
         "gpu_launches": launches,
         "clocks": clocks,
         "soak_steps": soak,
@@ -500,12 +645,82 @@ def run_ours(args, wl):
         dist.destroy_process_group()
 
 
+def run_update_scale(args, wl):
+    """UpdateGradScale of Algorithm 1 alone, element-wise, over the whole parameter set:
+    s = min(|g_small / (g_large + eps)|, s_max) with g_small = replica 1, g_large = replica 0
+    (12 bytes per parameter).  One process; a diagnostic of k_scale_elem, not a step."""
+    import torch
+
+    from paper_2603_18112_gb300 import build as B
+    from paper_2603_18112_gb300 import tula_ags as T
+    from paper_2603_18112_gb300 import workloads as W
+    if _dist()[0] > 1:
+        raise SystemExit("--step-kind update-scale runs on one GPU")
+    if not B.LIB.exists():
+        B.build()
+    T.lib()
+    K = max(2, wl.K)
+    buf = W.allocate(wl, "cuda", K=K)
+    W.fill_grads(buf, wl, step=1)
+    out = [torch.empty_like(t) for t in buf.w]
+    hp = T.tula_ags_default_hparams(K)
+    hp.granularity = T.TULA_SCALE_PER_ELEMENT
+    keep = T._tensor_ptrs(out)
+    hp.scale_elem = T.ctypes.cast(keep, T.c_void_p).value
+    stream = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    # marshalled once, as a training loop would keep them (the binding's per-call marshalling
+    # of 2 x n pointers costs more than the kernel on small sets)
+    n = wl.pset.n_tensors
+    g_small, g_large = T._tensor_ptrs(buf.g[1]), T._tensor_ptrs(buf.g[0])
+    numels, sp = T._numels(buf.g[0]), T._stream_ptr(stream)
+    lib = T.lib()
+
+    def call():
+        rc = lib.tula_ags_update_scale(g_small, g_large, numels, n, T.ctypes.byref(hp), sp)
+        if rc:
+            raise T.TulaError(rc, "tula_ags_update_scale")
+
+    with torch.cuda.stream(stream):
+        for _ in range(max(3, args.warmup)):
+            call()
+    stream.synchronize()
+    sampler = ClockSampler(0)
+    sampler.start()
+    launches0 = T.tula_ags_launch_count()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(args.steps):
+            call()
+        t1.record(stream)
+    stream.synchronize()
+    clocks = sampler.stop()
+    ms = t0.elapsed_time(t1) / args.steps
+    N = wl.pset.n_params
+    peak, peak_kind = _peaks()
+    gbs = scale_elem_bytes_per_param() * N / (ms / 1e3) / 1e9
+    print(json.dumps({
+        "metric": METRIC, "value": N / (ms / 1e3), "unit": UNIT, "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": _config(wl, wl.pset, "update-scale"),
+        "roofline": {"bound": "hbm", "kernel": "k_scale_elem (UpdateGradScale, element-wise)",
+                     "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
+                     "peak_kind": peak_kind, "traffic": None,
+                     "bytes_per_launch": scale_elem_bytes_per_param() * N, "ms_per_launch": ms},
+        "e2e": None, "gpu_launches": T.tula_ags_launch_count() - launches0, "clocks": clocks,
+    }), flush=True)
+
+
 def main():
     args = _args()
     from paper_2603_18112_gb300 import workloads as W
     wl = W.workload(args.workload)
     if args.impl == "reference":
         run_reference(args, wl)
+    elif args.step_kind == "update-scale":
+        run_update_scale(args, wl)
     else:
         run_ours(args, wl)
 

@@ -137,12 +137,12 @@ typedef struct tula_ags_hparams {
                                      not depend on it) */
     void *trace_events[5];        /* optional cudaEvent_t (NULL = none), recorded on `stream`:
                                      [0] before the reduction kernel(s), [1] after them,
-                                     [2] before the update kernel(s) (after a finish kernel
-                                     between the passes, which only LARS and per-element steps
-                                     have), [3] after the update kernel(s), [4] the end of the
-                                     step (after its last finish kernel).  A recorded event
-                                     keeps the next kernel from starting early, so steps that
-                                     record events run slightly slower. */
+                                     [2] after the pass-1 finish (before the update kernel),
+                                     [3] after the update kernel(s), [4] the end of the step
+                                     (after the finish that follows the update, when the step
+                                     has statistics or refreshes the gradscale).  A recorded
+                                     event keeps the next kernel from starting early, so steps
+                                     that record events run slightly slower. */
 } tula_ags_hparams;
 
 /* Fills *hp with the paper's defaults for K replicas: AGS, per tensor, automatic branch,

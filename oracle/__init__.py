@@ -89,6 +89,9 @@ def _load():
                                         ctypes.c_float, ctypes.c_float, ctypes.POINTER(_HP),
                                         f32p, pp, f64p, f64p]
         lib.oracle_ags_step.restype = ctypes.c_int
+        lib.oracle_ags_step_threads.argtypes = lib.oracle_ags_step.argtypes + [ctypes.c_int]
+        lib.oracle_ags_step_threads.restype = ctypes.c_int
+        lib.oracle_max_threads.restype = ctypes.c_int
         lib.oracle_layer_stats.argtypes = [pp, pp, ctypes.c_int, i64p, ctypes.c_int, f64p]
         lib.oracle_layer_stats.restype = ctypes.c_int
         lib.oracle_update_scale.argtypes = [pp, pp, i64p, ctypes.c_int, ctypes.c_float,
@@ -168,9 +171,15 @@ def new_state() -> np.ndarray:
     return np.zeros(STATE_LEN, dtype=np.float64)
 
 
+def max_threads() -> int:
+    """Threads ags_step(threads=...) can use (1 when the oracle was built without OpenMP)."""
+    return _load().oracle_max_threads()
+
+
 def ags_step(w, m, grads, lr, momentum, weight_decay, hp: OracleHP, scale=None,
-             scale_elem=None, state=None, want_stats=True):
-    """One optimizer step, in place.
+             scale_elem=None, state=None, want_stats=True, threads=None):
+    """One optimizer step, in place.  threads: run the per-tensor parts on that many threads
+    (the CPU baseline on all host cores); the result is the same bit for bit.
 
     w, m: lists of n float32 arrays (m may be None when hp.has_momentum is False).
     grads: K lists of n float32 arrays (replica k, tensor p); replica 0 receives
@@ -188,13 +197,16 @@ def ags_step(w, m, grads, lr, momentum, weight_decay, hp: OracleHP, scale=None,
     stats = np.zeros((n, STATS_LEN), dtype=np.float64) if want_stats else None
     chp = hp.to_c()
     m_list = m if (m is not None and hp.has_momentum) else [None] * n
-    rc = _load().oracle_ags_step(
-        _ptrs(w), _ptrs(m_list), _ptrs(flat_g), numel.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)),
-        n, lr, momentum, weight_decay, ctypes.byref(chp),
-        _fp(_f32(scale)) if scale is not None else None,
-        _ptrs(scale_elem) if scale_elem is not None else None,
-        state.ctypes.data_as(ctypes.POINTER(ctypes.c_double)),
-        stats.ctypes.data_as(ctypes.POINTER(ctypes.c_double)) if stats is not None else None)
+    args = (_ptrs(w), _ptrs(m_list), _ptrs(flat_g),
+            numel.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)), n, lr, momentum, weight_decay,
+            ctypes.byref(chp), _fp(_f32(scale)) if scale is not None else None,
+            _ptrs(scale_elem) if scale_elem is not None else None,
+            state.ctypes.data_as(ctypes.POINTER(ctypes.c_double)),
+            stats.ctypes.data_as(ctypes.POINTER(ctypes.c_double)) if stats is not None else None)
+    if threads is None:
+        rc = _load().oracle_ags_step(*args)
+    else:
+        rc = _load().oracle_ags_step_threads(*args, int(threads))
     if rc != 0:
         raise MemoryError("oracle_ags_step failed")
     return stats

@@ -20,8 +20,15 @@ def build_oracle(force: bool = False) -> Path:
     if not force and OUT.exists() and OUT.stat().st_mtime >= SRC.stat().st_mtime:
         return OUT
     tmp = OUT.with_suffix(f".{os.getpid()}.tmp")
-    cmd = [os.environ.get("CC", "gcc"), *CFLAGS, str(SRC), "-o", str(tmp), "-lm"]
-    subprocess.run(cmd, check=True)
+    cc = os.environ.get("CC", "gcc")
+    # OpenMP only spreads the per-tensor parts of oracle_ags_step_threads over threads; without
+    # it the same code runs on one thread.
+    for extra in (["-fopenmp"], []):
+        cmd = [cc, *CFLAGS, *extra, str(SRC), "-o", str(tmp), "-lm"]
+        if subprocess.run(cmd, capture_output=True).returncode == 0:
+            break
+    else:
+        subprocess.run(cmd, check=True)
     os.replace(tmp, OUT)
     return OUT
 

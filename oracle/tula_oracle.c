@@ -1,8 +1,10 @@
 /*
  * CPU oracle for the AGS optimizer step (Tula, arXiv 2603.18112).
  *
- * TEST INFRASTRUCTURE ONLY.  This file is a plain, slow, single-threaded
- * restatement of what the optimizer step computes, written from the paper:
+ * TEST INFRASTRUCTURE ONLY.  This file is a plain, slow restatement of what
+ * the optimizer step computes, written from the paper (single-threaded; the
+ * step's per-tensor parts can also run on several threads, for the CPU
+ * baseline on all host cores, with the same result):
  * the data-parallel mean of Eq. 1c, the gradient-variability metric of Eq. 5,
  * the scaled/unscaled branch and UpdateGradScale of Algorithm 1, the static
  * scaling function of Eq. 8, and the momentum-SGD + weight-decay update that
@@ -21,6 +23,9 @@
 #include <stddef.h>
 #include <stdint.h>
 #include <stdlib.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
 
 /* rule: how the per-tensor coefficient c_p is chosen */
 #define OR_RULE_AGS 0    /* Algorithm 1: c = gradscale[p] when Delta < delta, else 1 */
@@ -181,6 +186,106 @@ float oracle_scale_tensor(double s_small, double s_large, float eps, float s_max
     return (float)fmin(q, (double)s_max);
 }
 
+/* Steps 1-2 for tensor p: the norm of replica 0 (UpdateGradScale's small-batch gradient), the
+ * mean written over replica 0, and the norms of the mean and of w. */
+static void step_norms(float *const *w, float *const *g, const int64_t *numel, int n, int K, int p,
+                       const float **gp, double *sg, double *ss, double *sw)
+{
+    ss[p] = oracle_sqnorm(g[p], numel[p]);
+    for (int k = 0; k < K; ++k)
+        gp[k] = g[(int64_t)k * n + p];
+    oracle_replica_mean(gp, K, numel[p], g[p]);
+    sg[p] = oracle_sqnorm(g[p], numel[p]);
+    sw[p] = oracle_sqnorm(w[p], numel[p]);
+}
+
+/* Steps 4-5 for tensor p, once the branch is known: the coefficient, the update, the statistics
+ * row and UpdateGradScale. */
+static void step_update(float *const *w, float *const *m, float *const *g, const int64_t *numel,
+                        int p, float lr, float mu, float wd, const oracle_hp *hp, float *scale,
+                        float *const *scale_elem, int scaled, const double *sg, const double *ss,
+                        const double *sw, double *stats)
+{
+    int per_elem = hp->rule == OR_RULE_AGS && hp->granularity == OR_GRAN_ELEMENT;
+    float c = oracle_coefficient(hp->rule, scaled, scale ? scale[p] : 1.0f, hp->static_s,
+                                 hp->lars_trust, sw[p], sg[p]);
+    const float *ce = (per_elem && scaled) ? scale_elem[p] : NULL;
+    oracle_sgd_update(w[p], hp->has_momentum ? m[p] : NULL, g[p], numel[p], c, ce, lr, mu, wd);
+    if (per_elem)
+        c = scaled ? NAN : 1.0f; /* no single coefficient: reported as NaN when scaled */
+    float s_after = scale ? scale[p] : 0.0f;
+    if (hp->refresh_scale && hp->granularity == OR_GRAN_TENSOR && scale) {
+        s_after = oracle_scale_tensor(ss[p], sg[p], hp->eps, hp->s_max);
+        scale[p] = s_after;
+    }
+    if (stats) {
+        double *row = stats + (int64_t)p * OR_STATS_LEN;
+        row[0] = sw[p];
+        row[1] = sg[p];
+        row[2] = ss[p];
+        row[3] = sqrt(sw[p]);
+        row[4] = sqrt(sg[p]);
+        row[5] = oracle_trust_ratio(sw[p], sg[p]);
+        row[6] = (double)c;
+        row[7] = (double)s_after;
+    }
+}
+
+/* The step; threads > 1 runs the per-tensor parts of steps 1-2 and 4-5 on that many threads
+ * (OpenMP, when built with it).  Every tensor's arithmetic is the same whichever thread does
+ * it, and step 3 adds the norms in tensor order on one thread, so the result does not depend
+ * on the thread count. */
+static int ags_step(float *const *w, float *const *m, float *const *g, const int64_t *numel, int n,
+                    float lr, float mu, float wd, const oracle_hp *hp, float *scale,
+                    float *const *scale_elem, double *state, double *stats, int threads)
+{
+    int K = hp->K;
+    double *sg = calloc((size_t)n + 1, sizeof(double));
+    double *ss = calloc((size_t)n + 1, sizeof(double));
+    double *sw = calloc((size_t)n + 1, sizeof(double));
+    if (!sg || !ss || !sw) {
+        free(sg); free(ss); free(sw);
+        return -1;
+    }
+    int failed = 0;
+
+#pragma omp parallel for schedule(dynamic, 1) num_threads(threads > 0 ? threads : 1) reduction(|:failed)
+    for (int p = 0; p < n; ++p) {
+        const float **gp = malloc(sizeof(float *) * (size_t)(K > 0 ? K : 1));
+        if (!gp) {
+            failed = 1;
+            continue;
+        }
+        step_norms(w, g, numel, n, K, p, gp, sg, ss, sw);
+        free(gp);
+    }
+    if (failed) {
+        free(sg); free(ss); free(sw);
+        return -1;
+    }
+
+    /* step 3: |G|^2 in tensor order, Delta (Eq. 5), the branch (Algorithm 1) */
+    double g2 = 0.0;
+    for (int p = 0; p < n; ++p)
+        g2 = g2 + sg[p];
+    int64_t steps_done = (int64_t)state[1];
+    double dv = oracle_grad_variability(g2, state[0], steps_done);
+    int scaled = oracle_is_scaled(dv, hp->delta, hp->force_branch);
+
+#pragma omp parallel for schedule(dynamic, 1) num_threads(threads > 0 ? threads : 1)
+    for (int p = 0; p < n; ++p)
+        step_update(w, m, g, numel, p, lr, mu, wd, hp, scale, scale_elem, scaled, sg, ss, sw,
+                    stats);
+
+    state[0] = g2;
+    state[1] = (double)(steps_done + 1);
+    state[2] = dv;
+    state[3] = (double)scaled;
+
+    free(sg); free(ss); free(sw);
+    return 0;
+}
+
 /* One full optimizer step over n tensors, in the paper's order:
  *   1. mean of the K replicas (Eq. 1c), written over replica 0 when K > 1;
  *      |g_0|^2 is taken before it is overwritten
@@ -199,66 +304,26 @@ int oracle_ags_step(float *const *w, float *const *m, float *const *g, const int
                     int n, float lr, float mu, float wd, const oracle_hp *hp, float *scale,
                     float *const *scale_elem, double *state, double *stats)
 {
-    int K = hp->K;
-    double *sg = calloc((size_t)n + 1, sizeof(double));
-    double *ss = calloc((size_t)n + 1, sizeof(double));
-    double *sw = calloc((size_t)n + 1, sizeof(double));
-    const float **gp = malloc(sizeof(float *) * (size_t)(K > 0 ? K : 1));
-    if (!sg || !ss || !sw || !gp) {
-        free(sg); free(ss); free(sw); free(gp);
-        return -1;
-    }
+    return ags_step(w, m, g, numel, n, lr, mu, wd, hp, scale, scale_elem, state, stats, 1);
+}
 
-    for (int p = 0; p < n; ++p) {
-        ss[p] = oracle_sqnorm(g[p], numel[p]);
-        for (int k = 0; k < K; ++k)
-            gp[k] = g[(int64_t)k * n + p];
-        oracle_replica_mean(gp, K, numel[p], g[p]);
-        sg[p] = oracle_sqnorm(g[p], numel[p]);
-        sw[p] = oracle_sqnorm(w[p], numel[p]);
-    }
+/* The same step with its per-tensor parts on `threads` threads (the CPU baseline on all host
+ * cores); bitwise equal to oracle_ags_step. */
+int oracle_ags_step_threads(float *const *w, float *const *m, float *const *g, const int64_t *numel,
+                            int n, float lr, float mu, float wd, const oracle_hp *hp, float *scale,
+                            float *const *scale_elem, double *state, double *stats, int threads)
+{
+    return ags_step(w, m, g, numel, n, lr, mu, wd, hp, scale, scale_elem, state, stats, threads);
+}
 
-    double g2 = 0.0;
-    for (int p = 0; p < n; ++p)
-        g2 = g2 + sg[p];
-    int64_t steps_done = (int64_t)state[1];
-    double dv = oracle_grad_variability(g2, state[0], steps_done);
-    int scaled = oracle_is_scaled(dv, hp->delta, hp->force_branch);
-
-    for (int p = 0; p < n; ++p) {
-        int per_elem = hp->rule == OR_RULE_AGS && hp->granularity == OR_GRAN_ELEMENT;
-        float c = oracle_coefficient(hp->rule, scaled, scale ? scale[p] : 1.0f, hp->static_s,
-                                     hp->lars_trust, sw[p], sg[p]);
-        const float *ce = (per_elem && scaled) ? scale_elem[p] : NULL;
-        oracle_sgd_update(w[p], hp->has_momentum ? m[p] : NULL, g[p], numel[p], c, ce, lr, mu,
-                          wd);
-        if (per_elem)
-            c = scaled ? NAN : 1.0f; /* no single coefficient: reported as NaN when scaled */
-        float s_after = scale ? scale[p] : 0.0f;
-        if (hp->refresh_scale && hp->granularity == OR_GRAN_TENSOR && scale) {
-            s_after = oracle_scale_tensor(ss[p], sg[p], hp->eps, hp->s_max);
-            scale[p] = s_after;
-        }
-        if (stats) {
-            double *row = stats + (int64_t)p * OR_STATS_LEN;
-            row[0] = sw[p];
-            row[1] = sg[p];
-            row[2] = ss[p];
-            row[3] = sqrt(sw[p]);
-            row[4] = sqrt(sg[p]);
-            row[5] = oracle_trust_ratio(sw[p], sg[p]);
-            row[6] = (double)c;
-            row[7] = (double)s_after;
-        }
-    }
-
-    state[0] = g2;
-    state[1] = (double)(steps_done + 1);
-    state[2] = dv;
-    state[3] = (double)scaled;
-
-    free(sg); free(ss); free(sw); free(gp);
-    return 0;
+/* The number of threads oracle_ags_step_threads can use (1 when built without OpenMP). */
+int oracle_max_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
 }
 
 /* Per-layer statistics without an update: the mean of the K replicas is formed

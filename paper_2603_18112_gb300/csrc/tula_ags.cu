@@ -124,7 +124,8 @@ struct Table {
 
 struct Scalars {
     int K, rule, gran, force, refresh, mode, n_total, read_w;
-    int pow2K, evict_first, pad1, pad2;  // evict_first: TMA loads ask L2 to drop their lines first
+    int pow2K, evict_first, fin2, pad2;  // evict_first: TMA loads ask L2 to drop their lines first;
+                                         // fin2: a finish kernel follows the update
     float delta, eps, s_max, static_s, lars_trust, lr, mu, wd, invK, Kf;
     float *scale;
     double *state;
@@ -1267,68 +1268,100 @@ __global__ void __launch_bounds__(Ring1For<PR>::kThreads, 1)
 // After pass 1 of a step, one more warp forms |G|^2 from the global accumulator, then Delta
 // (Eq. 5) and the branch of Algorithm 1 (finalize_step).  No warp waits for another.
 
-// Per-tensor results after pass 1, by the whole warp that finished the tensor.  The square
-// roots are taken by lanes 0-2 in one fp64 sequence, and the two divisions likewise by lanes 0
-// and 1: GB300's FP64 pipe is slow, so the lanes share its latency instead of queueing behind it.
-__device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, double sw, float old) {
+// The square roots of three norms (lanes 0-2 in one fp64 sequence) and the two ratios of a
+// tensor (lanes 0 and 1): UpdateGradScale's |g_s| / (|g_l| + eps) and |w| / |gbar| (LARS, the
+// statistics).  GB300's FP64 pipe is slow, so the lanes share its latency instead of queueing
+// behind it.  Called by the whole warp; every lane gets every result.
+struct Norms {
+    double ng, ns, nw, q_scale, q_w;
+};
+__device__ __forceinline__ Norms tensor_norms(const Scalars &sc, double sg, double ss, double sw) {
     const int lane = threadIdx.x & 31;
     const double r = sqrt(lane == 0 ? sg : (lane == 1 ? ss : sw));
-    const double ng = __shfl_sync(kFull, r, 0), ns = __shfl_sync(kFull, r, 1),
-                 nw = __shfl_sync(kFull, r, 2);
-    // lane 0: UpdateGradScale's ratio |g_s| / (|g_l| + eps); lane 1: |w| / |gbar| (LARS and the
-    // statistics)
-    const double q = (lane == 0 ? ns : nw) / (lane == 0 ? ng + (double)sc.eps : ng);
-    const double q_scale = __shfl_sync(kFull, q, 0), q_w = __shfl_sync(kFull, q, 1);
+    Norms o;
+    o.ng = __shfl_sync(kFull, r, 0);
+    o.ns = __shfl_sync(kFull, r, 1);
+    o.nw = __shfl_sync(kFull, r, 2);
+    const double q = (lane == 0 ? o.ns : o.nw) / (lane == 0 ? o.ng + (double)sc.eps : o.ng);
+    o.q_scale = __shfl_sync(kFull, q, 0);
+    o.q_w = __shfl_sync(kFull, q, 1);
+    return o;
+}
+
+// The statistics row of a tensor from its squared norms (sw: |w|^2 before the update).
+__device__ __forceinline__ void stats_row(double *row, double sg, double ss, double sw,
+                                          const Norms &o) {
+    row[TULA_STAT_W_SQ] = sw;
+    row[TULA_STAT_G_SQ] = sg;
+    row[TULA_STAT_G0_SQ] = ss;
+    row[TULA_STAT_W_NORM] = o.nw;
+    row[TULA_STAT_G_NORM] = o.ng;
+    row[TULA_STAT_RATIO] = sg > 0.0 ? o.q_w : 0.0;
+}
+
+// Per-tensor results after pass 1, by the whole warp holding the tensor's norms.
+// tula_layer_stats and tula_ags_update_scale: everything here.  A step: what the update needs
+// (the coefficient c_p) and the norms, kept in tsum with the old gradscale; the square roots,
+// the statistics and UpdateGradScale follow the update (tensor_after_update), off the path
+// between the passes, except for LARS, whose coefficient is a ratio of norms.
+__device__ void tensor_done(const Scalars &sc, int tg, double sg, double ss, double sw, float old) {
+    const int lane = threadIdx.x & 31;
+    if (sc.mode == kModeScale || sc.mode == kModeStats || sc.rule == TULA_RULE_LARS) {
+        const Norms o = tensor_norms(sc, sg, ss, sw);
+        if (lane != 0) return;
+        if (sc.mode == kModeScale) {
+            // UpdateGradScale, g_0 = g_large, small = g_small: min(|g_s| / (|g_l| + eps), s_max)
+            sc.scale[tg] = (float)fmin(o.q_scale, (double)sc.s_max);
+            return;
+        }
+        if (sc.mode == kModeStats) {
+            double *row = sc.stats + (size_t)tg * TULA_STATS_LEN;
+            stats_row(row, sg, ss, sw, o);
+            row[TULA_STAT_COEF] = 0.0;
+            row[TULA_STAT_SCALE] = 0.0;
+            return;
+        }
+        // LARS (Sec. V-B): c_p = trust * |w| / |gbar|, every step (1 when either norm is 0)
+        sc.cand[tg] = (sw > 0.0 && sg > 0.0) ? (float)((double)sc.lars_trust * o.q_w) : 1.0f;
+    } else if (lane == 0) {
+        // the coefficient this tensor gets when the step is scaled (Algorithm 1, Eq. 8), before
+        // UpdateGradScale may overwrite gradscale
+        sc.cand[tg] = sc.rule == TULA_RULE_AGS ? old
+                      : (sc.rule == TULA_RULE_STATIC ? sc.static_s : 1.0f);
+    }
     if (lane != 0) return;
     double *T = sc.tsum + (size_t)tg * kTsum;
     T[0] = sg;
     T[1] = ss;
     T[2] = sw;
-    double *row = sc.stats ? sc.stats + (size_t)tg * TULA_STATS_LEN : nullptr;
-    if (sc.mode == kModeScale) {
-        // UpdateGradScale, g_0 = g_large, small = g_small: min(|g_s| / (|g_l| + eps), s_max)
-        sc.scale[tg] = (float)fmin(q_scale, (double)sc.s_max);
-        return;
-    }
-    if (sc.mode == kModeStats) {
-        row[TULA_STAT_W_SQ] = sw;
-        row[TULA_STAT_G_SQ] = sg;
-        row[TULA_STAT_G0_SQ] = ss;
-        row[TULA_STAT_W_NORM] = nw;
-        row[TULA_STAT_G_NORM] = ng;
-        row[TULA_STAT_RATIO] = sg > 0.0 ? q_w : 0.0;
-        row[TULA_STAT_COEF] = 0.0;
-        row[TULA_STAT_SCALE] = 0.0;
-        return;
-    }
-    // kModeStep: the coefficient this tensor gets when the step is scaled (Algorithm 1,
-    // Eq. 8) or always (LARS), before UpdateGradScale may overwrite gradscale.
-    float cand;
-    switch (sc.rule) {
-    case TULA_RULE_AGS: cand = old; break;
-    case TULA_RULE_STATIC: cand = sc.static_s; break;
-    case TULA_RULE_LARS:
-        cand = (sw > 0.0 && sg > 0.0) ? (float)((double)sc.lars_trust * q_w) : 1.0f;
-        break;
-    default: cand = 1.0f;
-    }
-    sc.cand[tg] = cand;
+    T[3] = (double)old;
+}
+
+// After the update of a step: the statistics row and UpdateGradScale of tensor t, from the
+// pass-1 norms kept in tsum and, when the update took it, |w|^2 from pass 2 (sw2).
+__device__ void tensor_after_update(const Scalars &sc, int t, double sw2, bool have_sw2) {
+    const int lane = threadIdx.x & 31;
+    const double *T = sc.tsum + (size_t)t * kTsum;
+    const double sg = T[0], ss = T[1], sw = have_sw2 ? sw2 : T[2];
+    const float old = (float)T[3];
+    const Norms o = tensor_norms(sc, sg, ss, sw);
+    if (lane != 0) return;
     float s_after = sc.scale ? old : 0.0f;
     if (sc.refresh && sc.scale) {
         // UpdateGradScale with g_small = replica 0 and g_large = the mean
-        s_after = (float)fmin(q_scale, (double)sc.s_max);
-        sc.scale[tg] = s_after;
+        s_after = (float)fmin(o.q_scale, (double)sc.s_max);
+        sc.scale[t] = s_after;
     }
-    if (row) {
-        row[TULA_STAT_G_SQ] = sg;
-        row[TULA_STAT_G0_SQ] = ss;
-        row[TULA_STAT_G_NORM] = ng;
-        row[TULA_STAT_SCALE] = (double)s_after;
-        if (sc.read_w) {
-            row[TULA_STAT_W_SQ] = sw;
-            row[TULA_STAT_W_NORM] = nw;
-            row[TULA_STAT_RATIO] = sg > 0.0 ? q_w : 0.0;
+    if (sc.stats) {
+        double *row = sc.stats + (size_t)t * TULA_STATS_LEN;
+        if (have_sw2 || sc.read_w) {
+            stats_row(row, sg, ss, sw, o);
+        } else {
+            row[TULA_STAT_G_SQ] = sg;
+            row[TULA_STAT_G0_SQ] = ss;
+            row[TULA_STAT_G_NORM] = o.ng;
         }
+        row[TULA_STAT_SCALE] = (double)s_after;
     }
 }
 
@@ -1391,22 +1424,9 @@ __device__ __forceinline__ double acc_read(unsigned long long *A, bool rearm) {
     return v[0];
 }
 
-// |w|^2 of tensor t from pass 2 into its statistics row (lanes 0 and 1 take the two square
-// roots in one instruction).
-__device__ __forceinline__ void w_stats(const Scalars &sc, int t, double sw, double sg) {
-    const int lane = threadIdx.x & 31;
-    const double r = sqrt(lane == 0 ? sw : sg);
-    const double nw = __shfl_sync(kFull, r, 0), ng = __shfl_sync(kFull, r, 1);
-    if (lane == 0) {
-        double *row = sc.stats + (size_t)t * TULA_STATS_LEN;
-        row[TULA_STAT_W_SQ] = sw;
-        row[TULA_STAT_W_NORM] = nw;
-        row[TULA_STAT_RATIO] = sg > 0.0 ? nw / ng : 0.0;
-    }
-}
-
 // NA = kAcc: after pass 1 (the pass-1 norms; in a step also the branch, which the update then
-// reads).  NA = 1: after pass 2 (|w|^2 for the statistics).
+// reads).  NA = 1: after the update of a step (its statistics and UpdateGradScale, with |w|^2
+// from pass 2 when the update took it).
 template <int NA>
 __global__ void __launch_bounds__(32 * kFinWarps) k_finish(const __grid_constant__ Scalars sc) {
     constexpr bool P1 = NA == kAcc;  // pass-1 accumulators
@@ -1443,8 +1463,9 @@ __global__ void __launch_bounds__(32 * kFinWarps) k_finish(const __grid_constant
         acc_to_double<kAcc>(w, v);
         tensor_done(sc, t, v[0], v[1], v[2], scale_old);
     } else {
-        const double sw = acc_read<kTCopies>(A2, true);
-        w_stats(sc, t, sw, sc.tsum[(size_t)t * kTsum + 0]);
+        const bool have_sw2 = sc.stats && !sc.read_w;  // the update's |w|^2 (k_update<..., SW>)
+        const double sw2 = have_sw2 ? acc_read<kTCopies>(A2, true) : 0.0;
+        tensor_after_update(sc, t, sw2, have_sw2);
     }
 }
 
@@ -1519,7 +1540,7 @@ __global__ void __launch_bounds__(Ring2::kThreads, 1)
     // Successors may start early only when the pass-2 finish follows (it waits
     // for this kernel); the next step's reduction, when it follows directly,
     // must start after this kernel has completed (see k_reduce).
-    if (SW) grid_launch_dependents();
+    if (sc.fin2) grid_launch_dependents();
     const bool early = !PE && tab.first;
     if (!early) grid_wait();
     uint64_t *full, *empty;
@@ -1719,11 +1740,25 @@ __global__ void __launch_bounds__(kScaleThreads)
         const float *a = ptr[0] + q.begin;
         const float *b = ptr[1] + q.begin;
         float *o = const_cast<float *>(ptr[2]) + q.begin;
-        for (int v = lane; v < nv; v += 32) {
-            const float4 x = __ldcs(reinterpret_cast<const float4 *>(a) + v);
-            const float4 y = __ldcs(reinterpret_cast<const float4 *>(b) + v);
-            st_stream(o + 4 * v, make_float4(scale1(x.x, y.x, sc), scale1(x.y, y.y, sc),
-                                             scale1(x.z, y.z, sc), scale1(x.w, y.w, sc)));
+        // Four float4 columns of each input per lane per step: eight 16-byte loads in flight
+        // per lane, which a plain-load streaming kernel needs to cover HBM latency.
+        for (int v0 = lane; v0 < nv; v0 += 4 * 32) {
+            float4 x[4], y[4];
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int v = v0 + 32 * u;
+                if (v < nv) {
+                    x[u] = __ldcs(reinterpret_cast<const float4 *>(a) + v);
+                    y[u] = __ldcs(reinterpret_cast<const float4 *>(b) + v);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < 4; ++u) {
+                const int v = v0 + 32 * u;
+                if (v < nv)
+                    st_stream(o + 4 * v, make_float4(scale1(x[u].x, y[u].x, sc), scale1(x[u].y, y[u].y, sc),
+                                                     scale1(x[u].z, y[u].z, sc), scale1(x[u].w, y[u].w, sc)));
+            }
         }
         const long long n = q.end - q.begin;
         for (long long j = 4 * (long long)nv + lane; j < n; j += 32)
@@ -2170,7 +2205,9 @@ int run_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mo
         dst[3] = per_elem ? hp->scale_elem[p] : nullptr;
     };
     const bool hm = mom_ptrs != nullptr;
-    const bool sw = hp->layer_stats != nullptr && !lars;
+    const bool sw = hp->layer_stats != nullptr && !lars;  // the update takes |w|^2
+    // The statistics and UpdateGradScale are finished after the update (k_finish<1>).
+    sc.fin2 = (hp->layer_stats != nullptr || hp->refresh_scale) ? 1 : 0;
     const int c2 = chunk2(hm, per_elem);
     sc.mode = kModeUpdate;
 #define TULA_UPD(HM, PE, SW)                                                                \
@@ -2186,7 +2223,7 @@ int run_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mo
 #undef TULA_UPD
     if (rc) return rc;
     record(hp->trace_events[3], s);
-    if (sw) rc = launch_finish<1>(n, sc, s);
+    if (sc.fin2) rc = launch_finish<1>(n, sc, s);
     if (rc) return rc;
     record(hp->trace_events[4], s);
     return TULA_OK;

@@ -18,12 +18,19 @@ def test_bytes_per_parameter(K):
     assert bench.step_min_bytes_per_param(K) == 4 * K + 16
     assert bench.step_min_bytes_per_param(K, read_w=True) == 4 * K + 20
     assert bench.step_min_bytes_per_param(K) <= bench.step_design_bytes_per_param(K)
+    # no momentum buffer: m is neither read nor written; a per-element gradscale is read
+    assert bench.pass2_bytes_per_param(False, True) == 16
+    assert bench.step_min_bytes_per_param(K, with_momentum=False) == 4 * K + 8
+    assert bench.step_min_bytes_per_param(K, per_element=True) == 4 * K + 20
+    assert bench.step_design_bytes_per_param(K, False, False, True) == \
+        bench.pass1_bytes_per_param(K) + 16
+    assert bench.scale_elem_bytes_per_param() == 12
 
 
 def test_step_kinds():
     # only LARS reads w in pass 1; only the refresh kind refreshes the gradscale every step
     assert bench.STEP_KINDS == {"ags": (False, False), "refresh": (False, True),
-                                "lars": (True, False)}
+                                "lars": (True, False), "update-scale": (False, False)}
     assert set(bench.STEP_KIND_TEXT) == set(bench.STEP_KINDS)
 
 
@@ -51,5 +58,6 @@ def test_reference_arm_prints_the_contract_line(kind):
     assert d["config"]["step"] == bench.STEP_KIND_TEXT[kind]
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
+    assert cb["cores"] == min(os.cpu_count(), bench.host_cores()) and cb["host_cpu_count"] == os.cpu_count()
     assert d["e2e"] == {"value": d["value"], "unit": bench.UNIT, "h2d_bytes_per_step": 0,
                         "d2h_bytes_per_step": 0}

@@ -570,3 +570,52 @@ def test_tensor_counts_around_a_finish_block(n, rule):
     for seed_step, mult in ((1, 1.0), (1, 1.0), (1, 2.0)):
         pair.step(seed_step, mult)
     assert pair.flags == [0, 1, 0]
+
+
+def test_checkpoint_and_resume_through_the_host():
+    """All AGS state lives in caller buffers (w, m, the gradscale, the step record), so a
+    checkpoint is a copy of them: 3 steps, the state copied to the host, a fresh optimizer step
+    (new device buffers, new workspace) built from those copies, 3 more steps -- bitwise the
+    same as 6 uninterrupted steps, statistics included, across both branches and a refresh."""
+    wl = W.workload("stress_k4", seed=151, factor_range=(0.1, 10.0), zero_patterns=False)
+    ps = _ragged_pset(K=4)
+    schedule = [(1, 1.0, True), (2, 1.0, False), (2, 1.0, False), (3, 2.0, False),
+                (4, 1.0, True), (4, 1.0, False)]
+
+    def fresh():
+        buf = W.allocate(wl, "cuda", K=4, pset=ps)
+        W.fill_state(buf, wl)
+        return buf
+
+    def run(buf, st, steps):
+        for seed_step, mult, refresh in steps:
+            W.fill_grads(buf, wl, step=seed_step, multiplier=mult)
+            st.step(wl.lr, wl.momentum, wl.weight_decay, refresh_scale=refresh)
+        torch.cuda.synchronize()
+
+    a = fresh()
+    st_a = T.AGSOptimizerStep(a.w, a.g, a.m, s_max=2.0)
+    run(a, st_a, schedule)
+
+    b = fresh()
+    st_b = T.AGSOptimizerStep(b.w, b.g, b.m, s_max=2.0)
+    run(b, st_b, schedule[:3])
+    ckpt = {"w": b.w_flat.cpu().numpy().copy(), "m": b.m_flat.cpu().numpy().copy(),
+            "state": st_b.state.cpu().numpy().copy(), "scale": st_b.scale.cpu().numpy().copy()}
+    del st_b, b
+    torch.cuda.empty_cache()
+
+    c = fresh()  # new buffers: the same shapes, contents replaced from the checkpoint
+    c.w_flat.copy_(torch.from_numpy(ckpt["w"]))
+    c.m_flat.copy_(torch.from_numpy(ckpt["m"]))
+    st_c = T.AGSOptimizerStep(c.w, c.g, c.m, s_max=2.0,
+                              scale=torch.from_numpy(ckpt["scale"]).cuda())
+    st_c.state.copy_(torch.from_numpy(ckpt["state"]))
+    torch.cuda.synchronize()
+    run(c, st_c, schedule[3:])
+
+    assert [int(x) for x in (st_a.state[3].item(), st_c.state[3].item())] == [1, 1]
+    assert st_a.state[1].item() == st_c.state[1].item() == 6.0
+    for x, y in ((a.w_flat, c.w_flat), (a.m_flat, c.m_flat), (a.g_flats[0], c.g_flats[0]),
+                 (st_a.state, st_c.state), (st_a.scale, st_c.scale), (st_a.stats, st_c.stats)):
+        assert torch.equal(x, y)

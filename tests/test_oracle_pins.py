@@ -441,3 +441,53 @@ def test_layer_stats_leaves_replicas_untouched():
     assert st[0].tolist() == [0.0] * 8
     mean = O.replica_mean([g[k][2] for k in range(3)])
     assert st[2, 1] == O.sqnorm(mean) and st[2, 0] == O.sqnorm(w[2])
+
+
+@pytest.mark.parametrize("rule,gran,refresh", [
+    (O.RULE_AGS, O.GRAN_TENSOR, True),
+    (O.RULE_AGS, O.GRAN_TENSOR, False),
+    (O.RULE_LARS, O.GRAN_TENSOR, False),
+    (O.RULE_AGS, O.GRAN_ELEMENT, False),
+])
+def test_threaded_oracle_is_bitwise_the_serial_one(rule, gran, refresh):
+    """The CPU baseline on all host cores runs the oracle's per-tensor parts on several threads;
+    the norms are still added in tensor order on one thread, so every output (w, m, the mean,
+    statistics, state, gradscale) must equal the single-threaded oracle's bit for bit, for any
+    thread count, over several steps of both branches."""
+    rng = np.random.default_rng(7)
+    numels = [int(x) for x in rng.integers(1, 3000, size=37)] + [0, 1, 40000]
+    K = 4
+
+    def inputs():
+        r = np.random.default_rng(8)
+        w = [r.standard_normal(n).astype(np.float32) for n in numels]
+        m = [(r.standard_normal(n) * 1e-3).astype(np.float32) for n in numels]
+        se = [r.uniform(0.5, 2.0, n).astype(np.float32) for n in numels]
+        return w, m, se
+
+    def grads(step, mult):
+        r = np.random.default_rng(100 + step)
+        return [[(r.standard_normal(n) * 1e-3 * mult).astype(np.float32) for n in numels]
+                for _ in range(K)]
+
+    runs = []
+    for threads in (None, 1, 2, 5, max(2, O.max_threads())):
+        w, m, se = inputs()
+        scale = np.linspace(0.5, 1.5, len(numels)).astype(np.float32)
+        state = O.new_state()
+        hp = O.OracleHP(K=K, rule=rule, granularity=gran, lars_trust=0.01)
+        out = []
+        for step, mult in ((1, 1.0), (1, 1.0), (2, 2.0)):
+            g = grads(step, mult)
+            hp.refresh_scale = refresh and step == 1
+            stats = O.ags_step(w, m, g, 0.1, 0.9, 5e-4, hp, scale=scale,
+                               scale_elem=se if gran == O.GRAN_ELEMENT else None, state=state,
+                               threads=threads)
+            out.append([np.concatenate(w), np.concatenate(m), np.concatenate(g[0]), stats,
+                        state.copy(), scale.copy()])
+        runs.append(out)
+    assert [int(s[4][3]) for s in runs[0]] == [0, 1, 0]  # both branches
+    for other in runs[1:]:
+        for a, b in zip(runs[0], other):
+            for x, y in zip(a, b):
+                assert np.array_equal(x, y, equal_nan=True)
