@@ -180,6 +180,37 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
                   float weight_decay, const tula_ags_hparams *hp, void *stream);
 
 /*
+ * A step sharded over ranks (one rank per GPU; the paper trains data-parallel with DDP, Sec.
+ * IV-A).  Each rank owns whole tensors and calls, with its own tensors only:
+ *   1. tula_ags_shard_reduce: pass 1 on its tensors -- the mean of its K replicas (Eq. 1c) and
+ *      their norms, kept in its workspace -- and its share of |G|^2 (Eq. 5) into g2_share;
+ *   2. an exchange of the shares that the caller makes (e.g. an all-reduce of the
+ *      TULA_G2_SHARE_WORDS uint64 words with an integer SUM over the ranks, in any order);
+ *   3. tula_ags_shard_update with the summed shares: Delta and the branch of Algorithm 1 from the
+ *      whole model's |G|^2, then the coefficients and the update of its tensors.
+ * A share is an exact integer: words 0-20 the 32-bit digits (from 2^-352) of the sum of this
+ * rank's tile partials of |gbar|^2 with carries in their high halves, word 21 the number of inf
+ * partials, word 22 the number of NaN partials, word 23 zero.  Integer addition has no order, so
+ * every rank takes the same |G|^2, Delta and branch, equal bit for bit to those of one
+ * tula_ags_step over all tensors (tiles are cut per tensor, so each tensor's norms are the same
+ * wherever it lives); the ranks together may span fewer than 2^31 pass-1 tiles.
+ * Arguments as tula_ags_step, with the rank's tensors; hp (workspace sized for the rank's
+ * tensors, state, scale, layer_stats) must be the same in both calls, and no other call may use
+ * the workspace between them.  g2_share, g2_total: device uint64 [TULA_G2_SHARE_WORDS], 8-byte
+ * aligned (TULA_ERR_ARG otherwise); g2_share is written, g2_total read.  Asynchronous on
+ * `stream`; the exchange must be ordered between the two calls.
+ */
+#define TULA_G2_SHARE_WORDS 24
+int tula_ags_shard_reduce(float *const *param_ptrs, float *const *grad_ptrs,
+                          float *const *mom_ptrs, const int64_t *numels, int n_tensors,
+                          float momentum, const tula_ags_hparams *hp, uint64_t *g2_share,
+                          void *stream);
+int tula_ags_shard_update(float *const *param_ptrs, float *const *grad_ptrs,
+                          float *const *mom_ptrs, const int64_t *numels, int n_tensors, float lr,
+                          float momentum, float weight_decay, const tula_ags_hparams *hp,
+                          const uint64_t *g2_total, void *stream);
+
+/*
  * Per-layer statistics without an update (read-only on every tensor): rows of
  * TULA_STATS_LEN fp64 as above, columns TULA_STAT_COEF and TULA_STAT_SCALE set to 0.
  * grad_ptrs[k*n + p] as in tula_ags_step.  stats_out: device fp64 [n_tensors][8].

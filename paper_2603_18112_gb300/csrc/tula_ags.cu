@@ -138,6 +138,7 @@ struct Scalars {
     double *tsum;              // [tensor][kTsum]: |gbar|^2, |g_0|^2, |w|^2
     float *cand;               // [tensor]: c_p of the scaled branch (AGS: the old gradscale)
     unsigned *tiles;           // [2 * pass]: next tile to claim, [2 * pass + 1]: CTAs finished
+    const unsigned long long *g2ext;  // a sharded step's |G|^2: the ranks' shares summed (or NULL)
 };
 
 // ----------------------------------------------------------------------------
@@ -1424,6 +1425,40 @@ __device__ __forceinline__ double acc_read(unsigned long long *A, bool rearm) {
     return v[0];
 }
 
+// A sharded step's share of |G|^2 (TULA_G2_SHARE_WORDS words): words 0 .. kAccDigits - 1 are the
+// digits of the global accumulator with its copies added, word kAccDigits counts inf partials
+// and the next one NaN partials, the rest are 0.  Every word adds as an integer, so the ranks'
+// shares combine by any integer sum, in any order, to the share of the whole step.
+static_assert(kAccDigits + 2 <= kAccWords && TULA_G2_SHARE_WORDS == kAccWords, "share layout");
+__device__ __forceinline__ double share_to_double(const unsigned long long *share) {
+    const int lane = threadIdx.x & 31;
+    unsigned long long w = lane < kAccWords ? __ldcg(share + lane) : 0ull;
+    const unsigned long long n_inf = __shfl_sync(kFull, w, kAccDigits);
+    const unsigned long long n_nan = __shfl_sync(kFull, w, kAccDigits + 1);
+    if (lane == kAccFlags) w = (n_nan ? 2ull : 0ull) | (n_inf ? 1ull : 0ull);
+    else if (lane >= kAccDigits) w = 0ull;
+    unsigned long long wi[1] = {w};
+    double v[1];
+    acc_to_double<1>(wi, v);
+    return v[0];
+}
+
+// Pass 1 of a sharded step, after the reduction: this rank's share of |G|^2 out of the global
+// accumulator, which is re-armed.  One warp.
+__global__ void __launch_bounds__(32) k_share(const __grid_constant__ Scalars sc,
+                                              unsigned long long *share) {
+    grid_wait();
+    const int lane = threadIdx.x & 31;
+    unsigned long long *const a[1] = {sc.gacc};
+    unsigned long long w[1];
+    acc_words<1, kGCopies>(a, true, w);
+    const unsigned long long flags = __shfl_sync(kFull, w[0], kAccFlags);
+    if (lane < kAccDigits) share[lane] = w[0];
+    else if (lane == kAccDigits) share[lane] = (flags & 1ull) ? 1ull : 0ull;
+    else if (lane == kAccDigits + 1) share[lane] = (flags & 2ull) ? 1ull : 0ull;
+    else if (lane < kAccWords) share[lane] = 0ull;
+}
+
 // NA = kAcc: after pass 1 (the pass-1 norms; in a step also the branch, which the update then
 // reads).  NA = 1: after the update of a step (its statistics and UpdateGradScale, with |w|^2
 // from pass 2 when the update took it).
@@ -1448,7 +1483,12 @@ __global__ void __launch_bounds__(32 * kFinWarps) k_finish(const __grid_constant
     const double g2_prev = step ? sc.state[TULA_STATE_G2_PREV] : 0.0;
     const double steps = step ? sc.state[TULA_STATE_STEPS] : 0.0;
     if (t == n) {  // the record and the branch
-        const double g2 = acc_read<kGCopies>(sc.gacc, true);
+        double g2;
+        if (sc.g2ext) {
+            g2 = share_to_double(sc.g2ext);
+        } else {
+            g2 = acc_read<kGCopies>(sc.gacc, true);
+        }
         if (lane == 0) finalize_step(sc, g2, g2_prev, steps);
         return;
     }
@@ -1999,26 +2039,26 @@ void record(void *ev, cudaStream_t s) {
 // Pass 1 (+ its finish) dispatched over the compile-time replica count.
 template <int KT, bool WM, bool RW, bool SS, bool PR, typename Fill>
 int run_reduce_k(int K, int n, const int64_t *numels, const Scalars &sc, int grid, cudaStream_t s,
-                 Fill fill, void *mid_event) {
+                 Fill fill, void *mid_event, bool finish) {
     const int chunk = chunk1(K, RW, SS);
     int rc = launch_streaming<P1<KT>::NP>(k_reduce<KT, WM, RW, SS, PR>, n, numels, chunk,
                                           Ring1For<PR>::kThreads, Ring1For<PR>::kSmemBytes, sc,
                                           grid, s, fill);
     if (rc) return rc;
     record(mid_event, s);
-    return launch_finish<kAcc>(n, sc, s);
+    return finish ? launch_finish<kAcc>(n, sc, s) : TULA_OK;
 }
 
 template <bool WM, bool RW, bool SS, bool PR, typename Fill>
 int run_reduce(int K, int n, const int64_t *numels, const Scalars &sc, int grid, cudaStream_t s,
-               Fill fill, void *mid_event = nullptr) {
+               Fill fill, void *mid_event = nullptr, bool finish = true) {
     switch (K) {
-    case 1: return run_reduce_k<1, false, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event);
-    case 2: return run_reduce_k<2, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event);
-    case 4: return run_reduce_k<4, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event);
-    case 8: return run_reduce_k<8, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event);
-    case 16: return run_reduce_k<16, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event);
-    default: return run_reduce_k<0, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event);
+    case 1: return run_reduce_k<1, false, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish);
+    case 2: return run_reduce_k<2, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish);
+    case 4: return run_reduce_k<4, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish);
+    case 8: return run_reduce_k<8, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish);
+    case 16: return run_reduce_k<16, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish);
+    default: return run_reduce_k<0, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish);
     }
 }
 
@@ -2154,11 +2194,17 @@ int check_step_args(float *const *param_ptrs, float *const *grad_ptrs, float *co
     return TULA_OK;
 }
 
+// Which part of a step run_step launches: all of it, or one half of a sharded step (pass 1 up to
+// this rank's share of |G|^2; then, from the ranks' shares summed, the rest).
+enum StepPart { kPartWhole = 0, kPartReduce = 1, kPartUpdate = 2 };
+
 // The step's launches, once its arguments (check_step_args) and its scratch `ws` (the caller's
 // workspace or the static array) have been accepted.
 int run_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mom_ptrs,
              const int64_t *numels, int n, float lr, float momentum, float weight_decay,
-             const tula_ags_hparams *hp, void *ws, const Plan &pl, void *stream) {
+             const tula_ags_hparams *hp, void *ws, const Plan &pl, void *stream,
+             StepPart part = kPartWhole, unsigned long long *share_out = nullptr,
+             const unsigned long long *g2_in = nullptr) {
     const int K = hp->K;
     const bool per_elem = hp->rule == TULA_RULE_AGS && hp->granularity == TULA_SCALE_PER_ELEMENT;
     int rc = TULA_OK;
@@ -2185,16 +2231,27 @@ int run_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mo
         dst[KS + 1] = nullptr;
     };
     record(hp->trace_events[0], s);
-    // Norms feeding a coefficient (LARS, UpdateGradScale) are taken precisely.
-    if (lars)
-        rc = run_reduce<true, true, false, true>(K, n, numels, sc, hp->grid_ctas, s, fill1,
-                                                 hp->trace_events[1]);
-    else if (hp->refresh_scale)
-        rc = run_reduce<true, false, false, true>(K, n, numels, sc, hp->grid_ctas, s, fill1,
-                                                  hp->trace_events[1]);
-    else
-        rc = run_reduce<true, false, false, false>(K, n, numels, sc, hp->grid_ctas, s, fill1,
-                                                   hp->trace_events[1]);
+    if (part == kPartUpdate) {
+        // the ranks' shares summed give |G|^2; the local accumulators the tensors' norms
+        sc.g2ext = g2_in;
+        record(hp->trace_events[1], s);
+        rc = launch_finish<kAcc>(n, sc, s);
+        sc.g2ext = nullptr;
+    } else {
+        const bool fin = part == kPartWhole;
+        // Norms feeding a coefficient (LARS, UpdateGradScale) are taken precisely.
+        if (lars)
+            rc = run_reduce<true, true, false, true>(K, n, numels, sc, hp->grid_ctas, s, fill1,
+                                                     hp->trace_events[1], fin);
+        else if (hp->refresh_scale)
+            rc = run_reduce<true, false, false, true>(K, n, numels, sc, hp->grid_ctas, s, fill1,
+                                                      hp->trace_events[1], fin);
+        else
+            rc = run_reduce<true, false, false, false>(K, n, numels, sc, hp->grid_ctas, s, fill1,
+                                                       hp->trace_events[1], fin);
+        if (rc == TULA_OK && part == kPartReduce)
+            return launch_pdl(k_share, 1, 32, 0, s, sc, share_out);
+    }
     if (rc) return rc;
     record(hp->trace_events[2], s);
 
@@ -2243,6 +2300,36 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
     if (rc) return rc;
     return run_step(param_ptrs, grad_ptrs, mom_ptrs, numels, n_tensors, lr, momentum,
                     weight_decay, hp, hp->workspace, pl, stream);
+}
+
+int tula_ags_shard_reduce(float *const *param_ptrs, float *const *grad_ptrs,
+                          float *const *mom_ptrs, const int64_t *numels, int n_tensors,
+                          float momentum, const tula_ags_hparams *hp, uint64_t *g2_share,
+                          void *stream) {
+    Plan pl;
+    int rc = check_step_args(param_ptrs, grad_ptrs, mom_ptrs, numels, n_tensors, momentum, hp, &pl);
+    if (rc) return rc;
+    if (!g2_share || (reinterpret_cast<uintptr_t>(g2_share) & 7u)) return TULA_ERR_ARG;
+    rc = check_ws(hp->workspace, hp->workspace_bytes, n_tensors, pl);
+    if (rc) return rc;
+    return run_step(param_ptrs, grad_ptrs, mom_ptrs, numels, n_tensors, 0.f, momentum, 0.f, hp,
+                    hp->workspace, pl, stream, kPartReduce,
+                    reinterpret_cast<unsigned long long *>(g2_share), nullptr);
+}
+
+int tula_ags_shard_update(float *const *param_ptrs, float *const *grad_ptrs,
+                          float *const *mom_ptrs, const int64_t *numels, int n_tensors, float lr,
+                          float momentum, float weight_decay, const tula_ags_hparams *hp,
+                          const uint64_t *g2_total, void *stream) {
+    Plan pl;
+    int rc = check_step_args(param_ptrs, grad_ptrs, mom_ptrs, numels, n_tensors, momentum, hp, &pl);
+    if (rc) return rc;
+    if (!g2_total || (reinterpret_cast<uintptr_t>(g2_total) & 7u)) return TULA_ERR_ARG;
+    rc = check_ws(hp->workspace, hp->workspace_bytes, n_tensors, pl);
+    if (rc) return rc;
+    return run_step(param_ptrs, grad_ptrs, mom_ptrs, numels, n_tensors, lr, momentum,
+                    weight_decay, hp, hp->workspace, pl, stream, kPartUpdate, nullptr,
+                    reinterpret_cast<const unsigned long long *>(g2_total));
 }
 
 int tula_layer_stats(const float *const *param_ptrs, const float *const *grad_ptrs, int K,
@@ -2317,7 +2404,7 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
         dst[2] = g_small[p];
     };
     return run_reduce_k<1, false, false, true, true>(1, n, numels, sc, hp->grid_ctas, s, fill,
-                                                     nullptr);
+                                                     nullptr, true);
 }
 
 const char *tula_ags_error_string(int code) {

@@ -26,6 +26,7 @@ TULA_RULE_AGS, TULA_RULE_NONE, TULA_RULE_LARS, TULA_RULE_STATIC = 0, 1, 2, 3
 TULA_SCALE_PER_TENSOR, TULA_SCALE_PER_ELEMENT = 0, 1
 TULA_BRANCH_AUTO, TULA_BRANCH_SCALED, TULA_BRANCH_UNSCALED = 0, 1, 2
 TULA_STATE_LEN, TULA_STATS_LEN = 4, 8
+TULA_G2_SHARE_WORDS = 24
 (TULA_STAT_W_SQ, TULA_STAT_G_SQ, TULA_STAT_G0_SQ, TULA_STAT_W_NORM, TULA_STAT_G_NORM,
  TULA_STAT_RATIO, TULA_STAT_COEF, TULA_STAT_SCALE) = range(8)
 
@@ -91,11 +92,15 @@ def lib() -> ctypes.CDLL:
                                            ctypes.POINTER(c_int)]
     L.tula_ags_check_wait_timeout.argtypes = [c_void_p, c_size_t, c_void_p]
     L.tula_ags_static_scratch_error.argtypes = [c_void_p, ctypes.POINTER(c_int)]
+    L.tula_ags_shard_reduce.argtypes = [pp, pp, pp, i64p, c_int, c_float, hpp, c_void_p, c_void_p]
+    L.tula_ags_shard_update.argtypes = [pp, pp, pp, i64p, c_int, c_float, c_float, c_float, hpp,
+                                        c_void_p, c_void_p]
     L.tula_ags_static_scratch_check_wait_timeout.argtypes = [c_void_p]
     for name in ("tula_ags_workspace_size", "tula_ags_step", "tula_layer_stats",
                  "tula_ags_update_scale", "tula_ags_plan_chunks", "tula_ags_step_static_scratch",
                  "tula_ags_workspace_error", "tula_ags_check_wait_timeout",
-                 "tula_ags_static_scratch_error", "tula_ags_static_scratch_check_wait_timeout"):
+                 "tula_ags_static_scratch_error", "tula_ags_static_scratch_check_wait_timeout",
+                 "tula_ags_shard_reduce", "tula_ags_shard_update"):
         getattr(L, name).restype = c_int
     _lib = L
     return L
@@ -371,3 +376,49 @@ class AGSOptimizerStep:
         _check(rc, "tula_ags_step")
 
     __call__ = step
+
+    # -- a step sharded over ranks: this object holds one rank's tensors --------------------
+
+    def new_g2_share(self) -> torch.Tensor:
+        """A device buffer for a share of |G|^2 (TULA_G2_SHARE_WORDS uint64, held as int64: the
+        integer sums of the exchange wrap the same way)."""
+        return torch.zeros(TULA_G2_SHARE_WORDS, dtype=torch.int64, device=self.params[0].device)
+
+    def shard_reduce(self, momentum, g2_share: torch.Tensor, refresh_scale=False,
+                     stream=None) -> None:
+        """Pass 1 on this rank's tensors; its share of |G|^2 into g2_share."""
+        self.hp.refresh_scale = 1 if refresh_scale else 0
+        rc = lib().tula_ags_shard_reduce(self._p, self._g, self._m, self._numels, self.n, momentum,
+                                         ctypes.byref(self.hp), c_void_p(g2_share.data_ptr()),
+                                         _stream_ptr(stream))
+        _check(rc, "tula_ags_shard_reduce")
+
+    def shard_update(self, lr, momentum, weight_decay, g2_total: torch.Tensor,
+                     refresh_scale=False, stream=None) -> None:
+        """The rest of the step on this rank's tensors, from every rank's share summed."""
+        self.hp.refresh_scale = 1 if refresh_scale else 0
+        rc = lib().tula_ags_shard_update(self._p, self._g, self._m, self._numels, self.n, lr,
+                                         momentum, weight_decay, ctypes.byref(self.hp),
+                                         c_void_p(g2_total.data_ptr()), _stream_ptr(stream))
+        _check(rc, "tula_ags_shard_update")
+
+
+def combine_g2_shares(share: torch.Tensor, group=None) -> torch.Tensor:
+    """The exchange of a sharded step: every rank's share of |G|^2 summed, in place, over the
+    torch.distributed group (an integer SUM, exact and independent of the reduction order).
+    Without an initialised process group or with one rank, the share is the total."""
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size(group) > 1:
+        dist.all_reduce(share, op=dist.ReduceOp.SUM, group=group)
+    return share
+
+
+def sharded_step(step: AGSOptimizerStep, lr, momentum, weight_decay, group=None,
+                 refresh_scale=False, share=None) -> torch.Tensor:
+    """One step sharded over the group's ranks: shard_reduce, the exchange, shard_update, all
+    on the current stream.  Returns the summed share."""
+    share = step.new_g2_share() if share is None else share
+    step.shard_reduce(momentum, share, refresh_scale)
+    combine_g2_shares(share, group)
+    step.shard_update(lr, momentum, weight_decay, share, refresh_scale)
+    return share

@@ -172,3 +172,21 @@ def test_binding_refuses_replica_lists_that_do_not_match(lib):
         T.AGSOptimizerStep(params, [[torch.zeros(4)]])
     with pytest.raises(ValueError):
         T.AGSOptimizerStep(params, [])
+
+
+def test_sharded_step_argument_errors(lib):
+    """The two halves of a sharded step check their arguments like tula_ags_step, and the share
+    pointer (NULL or not 8-byte aligned) before any CUDA call."""
+    P = ctypes.c_void_p
+    ptrs = (P * 4)(*[0x10000 * (i + 1) for i in range(4)])
+    numels = (ctypes.c_int64 * 2)(5, 7)
+    hp = T.tula_ags_default_hparams(1)
+    hp.scale, hp.state, hp.workspace, hp.workspace_bytes = 0x20000, 0x30000, 0x40000, 1 << 30
+    for share in (None, 0x50004):
+        assert lib.tula_ags_shard_reduce(ptrs, ptrs, ptrs, numels, 2, 0.9, ctypes.byref(hp),
+                                         share, None) == T.TULA_ERR_ARG
+        assert lib.tula_ags_shard_update(ptrs, ptrs, ptrs, numels, 2, 0.1, 0.9, 0.0,
+                                         ctypes.byref(hp), share, None) == T.TULA_ERR_ARG
+    hp.state = 0
+    assert lib.tula_ags_shard_reduce(ptrs, ptrs, ptrs, numels, 2, 0.9, ctypes.byref(hp),
+                                     0x50000, None) == T.TULA_ERR_ARG

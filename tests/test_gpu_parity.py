@@ -619,3 +619,48 @@ def test_checkpoint_and_resume_through_the_host():
     for x, y in ((a.w_flat, c.w_flat), (a.m_flat, c.m_flat), (a.g_flats[0], c.g_flats[0]),
                  (st_a.state, st_c.state), (st_a.scale, st_c.scale), (st_a.stats, st_c.stats)):
         assert torch.equal(x, y)
+
+
+@pytest.mark.parametrize("name,rule", [("resnet50", T.TULA_RULE_AGS), ("resnet18", T.TULA_RULE_LARS),
+                                       ("ragged_k4", T.TULA_RULE_AGS)])
+def test_sharded_step_equals_the_whole_step(name, rule):
+    """A step sharded over two ranks (each owning whole tensors) run on one GPU, one shard after
+    the other: each rank's pass 1 exports its share of |G|^2, the shares are summed as integers,
+    and each rank finishes from the sum.  Tiles are cut per tensor and the sums are exact, so the
+    mean, every norm, |G|^2, Delta, the branch, w, m and the gradscale equal those of one step
+    over all tensors bit for bit -- whichever order the shares are added in."""
+    if name == "ragged_k4":
+        wl = W.workload("stress_k4", seed=161, factor_range=(0.1, 10.0), zero_patterns=False)
+        ps = _ragged_pset(K=4)
+    else:
+        wl, ps = W.workload(name), None
+    K = 4 if ps is not None else wl.K
+    a, b = (W.allocate(wl, "cuda", K=K, pset=ps) for _ in range(2))
+    for buf in (a, b):
+        W.fill_state(buf, wl)
+    n = a.pset.n_tensors
+    cut = n // 2 + 1
+    kw = dict(s_max=2.0, rule=rule, lars_trust=0.01)
+    whole = T.AGSOptimizerStep(a.w, a.g, a.m, **kw)
+    ranks = [T.AGSOptimizerStep(b.w[lo:hi], [b.g[k][lo:hi] for k in range(K)], b.m[lo:hi], **kw)
+             for lo, hi in ((0, cut), (cut, n))]
+    shares = [r.new_g2_share() for r in ranks]
+    for i, (seed_step, mult) in enumerate(((1, 1.0), (1, 1.0), (1, 2.0), (2, 1.0))):
+        refresh = rule == T.TULA_RULE_AGS and i == 0
+        for buf in (a, b):
+            W.fill_grads(buf, wl, step=seed_step, multiplier=mult)
+        whole.step(wl.lr, wl.momentum, wl.weight_decay, refresh_scale=refresh)
+        for r, sh in zip(ranks, shares):
+            r.shard_reduce(wl.momentum, sh, refresh_scale=refresh)
+        total = shares[1] + shares[0] if i % 2 else shares[0] + shares[1]  # either order
+        for r in ranks:
+            r.shard_update(wl.lr, wl.momentum, wl.weight_decay, total, refresh_scale=refresh)
+        torch.cuda.synchronize()
+        where = f"{name} step {i + 1}"
+        for r in ranks:
+            assert torch.equal(r.state, whole.state), where + " state"
+        assert torch.equal(torch.cat([r.stats for r in ranks]), whole.stats), where + " stats"
+        assert torch.equal(torch.cat([r.scale for r in ranks]), whole.scale), where + " scale"
+        for x, y in ((a.w_flat, b.w_flat), (a.m_flat, b.m_flat), (a.g_flats[0], b.g_flats[0])):
+            assert torch.equal(x, y), where
+    assert [int(v) for v in (whole.state[1].item(),)] == [4]
