@@ -621,6 +621,9 @@ def run_ours(args, wl):
                      "traffic": traffic, "bytes_per_launch": p1_bytes,
                      "ms_per_launch": p1_avg_ms},
         "update_pass": {"kernel": "k_update (scaled momentum-SGD)", "bytes_per_launch": p2_bytes,
+                        "traffic": _ncu_traffic("k_update" + ("_per_element" if per_elem else "")
+                                                + ("" if args.momentum else "_no_momentum"),
+                                                wl.name, N),
                         "ms_per_launch": p2_avg_ms,
                         "achieved_gbs": p2_bytes / (p2_avg_ms / 1e3) / 1e9,
                         "frac": p2_bytes / (p2_avg_ms / 1e3) / 1e9 / peak},

@@ -151,7 +151,7 @@ typedef struct tula_ags_hparams {
 void tula_ags_default_hparams(tula_ags_hparams *hp, int K);
 
 /* Bytes of workspace needed for this list of tensor sizes and K replicas (host only): about
- * 3.1 KB per tensor (accumulators and per-tensor sums), whatever the tensors' sizes. */
+ * 1.6 KB per tensor (accumulators and per-tensor sums), whatever the tensors' sizes. */
 int tula_ags_workspace_size(const int64_t *numels, int n_tensors, int K, size_t *bytes);
 
 /*
@@ -250,8 +250,8 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
  * TULA_STATIC_SCRATCH_BYTES (16 MiB) inside this library.  Every GPU that loads the library holds
  * that array until the process exits.  hp->workspace and hp->workspace_bytes are ignored.
  *
- * Limit: the scratch a tensor list needs (tula_ags_workspace_size) is about 3.1 KB per tensor,
- * whatever the tensors' sizes and K: up to 5,397 tensors.  A longer list is rejected with
+ * Limit: the scratch a tensor list needs (tula_ags_workspace_size) is about 1.6 KB per tensor,
+ * whatever the tensors' sizes and K: up to 10,670 tensors.  A longer list is rejected with
  * TULA_ERR_SCRATCH_LIMIT before anything is enqueued.
  *
  * Set-up: every call looks up the array's device address in the current device's context

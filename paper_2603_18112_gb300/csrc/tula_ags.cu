@@ -76,17 +76,13 @@ struct Ring {
         return (kStageBytes / (4 * streams)) / 128 * 128;
     }
 };
-// Pass 1 streams K (+1, +2) tensors and little arithmetic: large copies, few
-// consumers.  Pass 2 does ~11 flops per element over 3-4 streams: its
-// consumers, not HBM, set the pace with three warps, so it runs four.
-using Ring1 = Ring<36, 6, 3>;
-// The precise pass 1 (float-float squares) spends ~13 dependent FP32 instructions per element
-// and norm: six consumers, two per scheduler, hide that latency.  Same stages, same tiles.
-using Ring1P = Ring<36, 6, 6>;
-template <bool PR>
-using Ring1For = std::conditional_t<PR, Ring1P, Ring1>;
-static_assert(Ring1P::kStageBytes == Ring1::kStageBytes && Ring1P::kStages == Ring1::kStages,
-              "both pass-1 rings cut the same tiles");
+// Pass 1 streams K (+1, +2) tensors through 36 KB stages.  Six consumer warps, two per
+// scheduler: the precise norms spend ~13 dependent FP32 instructions per element and norm, and
+// the default ones add their tile sums into the accumulators at the end of each batch; with
+// three warps the reduction ran 0.8 % slower alone (the same step time).
+using Ring1 = Ring<36, 6, 6>;
+// Pass 2 does ~11 flops per element over 3-4 streams: with three consumer warps they, not HBM,
+// set its pace, so it runs four.
 using Ring2 = Ring<24, 8, 4>;
 constexpr int kDynTiles = 64;            // tiles per CTA from which a launch claims its tiles
 constexpr unsigned kClaim = 4;           // tiles per claim
@@ -377,7 +373,7 @@ constexpr int kAccDigits = 21;
 constexpr int kAccWords = 24;             // digits, two spare words, the flags
 constexpr int kAccFlags = kAccWords - 1;  // bit 0: an inf partial, bit 1: a NaN partial
 constexpr int kAccBase = -352;
-constexpr int kTCopies = 4;               // copies of each per-tensor accumulator
+constexpr int kTCopies = 2;               // copies of each per-tensor accumulator
 constexpr int kGCopies = 8;               // copies of the |G|^2 accumulator
 static_assert(kAccDigits <= kAccFlags && kAccWords <= 32, "one word per lane");
 static_assert((kTCopies & (kTCopies - 1)) == 0 && (kGCopies & (kGCopies - 1)) == 0, "powers of 2");
@@ -1129,7 +1125,7 @@ __device__ __noinline__ void add_tile_now(const Scalars &sc, int tg, const float
 }
 
 template <int KT, bool WM, bool RW, bool SS, bool PR>
-__global__ void __launch_bounds__(Ring1For<PR>::kThreads, 1)
+__global__ void __launch_bounds__(Ring1::kThreads, 1)
     k_reduce(const __grid_constant__ Table<P1<KT>::NP> tab, const __grid_constant__ Scalars sc) {
     constexpr int KS = P1<KT>::KS;
     constexpr int NSMAX = KS + 2;
@@ -1149,7 +1145,7 @@ __global__ void __launch_bounds__(Ring1For<PR>::kThreads, 1)
     if (!early) grid_wait();
     uint64_t *full, *empty;
     int *stage_tile;
-    using R1 = Ring1For<PR>;
+    using R1 = Ring1;
     ring_setup<R1>(smem, full, empty, stage_tile);
     const int js = static_tiles(tab.nc);
     const uint32_t ring = smem_addr(smem);
@@ -2042,7 +2038,7 @@ int run_reduce_k(int K, int n, const int64_t *numels, const Scalars &sc, int gri
                  Fill fill, void *mid_event, bool finish) {
     const int chunk = chunk1(K, RW, SS);
     int rc = launch_streaming<P1<KT>::NP>(k_reduce<KT, WM, RW, SS, PR>, n, numels, chunk,
-                                          Ring1For<PR>::kThreads, Ring1For<PR>::kSmemBytes, sc,
+                                          Ring1::kThreads, Ring1::kSmemBytes, sc,
                                           grid, s, fill);
     if (rc) return rc;
     record(mid_event, s);
