@@ -533,14 +533,26 @@ def run_ours(args, wl):
     launches = T.tula_ags_launch_count() - launches0
     # Host time per call: 50 steps issued after a synchronize, timed on the host up to the
     # return of the last call (the launch queue holds them all, so the host never waits on
-    # the GPU unless it is the faster side).
-    torch.cuda.synchronize()
-    h0 = time.perf_counter()
-    with torch.cuda.stream(stream):
-        for _ in range(50):
-            one_step()
-    host_us = (time.perf_counter() - h0) / 50 * 1e6
-    torch.cuda.synchronize()
+    # the GPU unless it is the faster side).  Once through the plan the timed steps use, once
+    # through tula_ags_step, which checks every pointer and builds the launch tables per call.
+    def host_us_per_call(fn):
+        torch.cuda.synchronize()
+        h0 = time.perf_counter()
+        with torch.cuda.stream(stream):
+            for _ in range(50):
+                fn()
+        us = (time.perf_counter() - h0) / 50 * 1e6
+        torch.cuda.synchronize()
+        return us
+
+    host_us = host_us_per_call(one_step)
+    direct = T.AGSOptimizerStep(buf.w, buf.g, buf.m if args.momentum else None, s_max=wl.smax,
+                                rule=step.hp.rule, lars_trust=LARS_TRUST,
+                                granularity=step.hp.granularity, scale_elem=scale_elem,
+                                plan=False)
+    host_us_direct = host_us_per_call(
+        lambda: direct.step(wl.lr, mu, wl.weight_decay, refresh_scale=refresh, stream=stream))
+    del direct
     peak, peak_kind = _peaks()
     secondary = (secondary_record(SECONDARY, args, kind, stream, peak)
                  if args.secondary and wl.name != SECONDARY and not per_elem and args.momentum
@@ -636,6 +648,7 @@ def run_ours(args, wl):
                      "design_gbs": sdes * N / (ms_per_step / 1e3) / 1e9},
         "e2e": e2e,
         "host_us_per_call": host_us,
+        "host_us_per_call_direct": host_us_direct,
         "secondary": [secondary] if secondary else [],
         "gpu_launches": launches,
         "clocks": clocks,

@@ -71,6 +71,8 @@ extern "C" {
 #define TULA_ERR_UNSUPPORTED (-4) /* a valid but unimplemented combination of options */
 #define TULA_ERR_SCRATCH_LIMIT (-5) /* tula_ags_step_static_scratch: the tensor list needs more
                                        scratch than TULA_STATIC_SCRATCH_BYTES */
+#define TULA_ERR_NO_MEMORY (-6)   /* host memory for launch tables or a plan could not be
+                                     allocated; nothing was enqueued */
 
 #define TULA_MAX_K 16
 
@@ -178,6 +180,36 @@ int tula_ags_workspace_size(const int64_t *numels, int n_tensors, int K, size_t 
 int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mom_ptrs,
                   const int64_t *numels, int n_tensors, float lr, float momentum,
                   float weight_decay, const tula_ags_hparams *hp, void *stream);
+
+/*
+ * A plan: the same step as tula_ags_step for a training loop that steps one fixed set of tensors
+ * again and again.  tula_ags_plan_create checks the sizes and pointers once and copies them;
+ * each tula_ags_plan_step then checks only hp and the scalars, and the launch tables (sizes and
+ * pointers of up to ~31 KB per kernel launch) are built by the first step of each kernel variant
+ * and reused by every later one.  Results are those of tula_ags_step bit for bit.
+ *   tula_ags_plan_create: arguments as tula_ags_step.  Of hp only K and scale_elem are read:
+ *     the per-element gradscale buffers, when given, are copied with the rest and are the ones
+ *     every step of the plan uses (a step with PER_ELEMENT needs them).  The arrays and hp may
+ *     be freed on return; the tensors must stay allocated until the plan is destroyed.  Binds
+ *     the plan to the current CUDA device.  *plan_out receives the plan (NULL on error).
+ *     Errors: TULA_ERR_ARG (as tula_ags_step, or plan_out NULL), TULA_ERR_CUDA (no current
+ *     device), TULA_ERR_NO_MEMORY.  Allocates host memory only.
+ *   tula_ags_plan_step: lr, momentum, weight_decay and hp as tula_ags_step; hp->K must be the
+ *     plan's, and hp->scale_elem is ignored.  Every other field (rule, granularity, branch,
+ *     refresh, scale, state, layer_stats, workspace, grid_ctas, trace_events) may change from
+ *     one call to the next.  Momentum != 0 needs a plan created with momentum buffers.  Errors
+ *     as tula_ags_step, and TULA_ERR_ARG when the current device is not the plan's.
+ *   tula_ags_plan_destroy: frees the plan (NULL is a no-op).  Launches already issued do not
+ *     use it, so it may be destroyed as soon as the last tula_ags_plan_step has returned.
+ * A plan is not thread-safe: one host thread at a time may call tula_ags_plan_step on it.
+ */
+typedef struct tula_ags_plan tula_ags_plan;
+int tula_ags_plan_create(float *const *param_ptrs, float *const *grad_ptrs,
+                         float *const *mom_ptrs, const int64_t *numels, int n_tensors,
+                         const tula_ags_hparams *hp, tula_ags_plan **plan_out);
+int tula_ags_plan_step(tula_ags_plan *plan, float lr, float momentum, float weight_decay,
+                       const tula_ags_hparams *hp, void *stream);
+int tula_ags_plan_destroy(tula_ags_plan *plan);
 
 /*
  * A step sharded over ranks (one rank per GPU; the paper trains data-parallel with DDP, Sec.

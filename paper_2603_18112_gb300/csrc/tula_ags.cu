@@ -51,6 +51,7 @@
 #include <cstring>
 #include <memory>
 #include <mutex>
+#include <new>
 #include <type_traits>
 #include <utility>
 #include <vector>
@@ -1937,48 +1938,80 @@ int launch_pdl(void (*kernel)(KArgs...), int grid, int threads, int smem, cudaSt
     return TULA_OK;
 }
 
+// The launch tables of a plan (tula_ags_plan_create): for each kernel instantiation and tile
+// size, its parameter blocks, built by the first call that launches them and reused by every
+// later one (they hold only sizes and pointers, which a plan fixes).
+struct TableCache {
+    struct Entry {
+        const void *kernel;
+        int chunk;
+        std::vector<std::shared_ptr<const void>> blocks;
+    };
+    std::vector<Entry> entries;
+    const std::vector<std::shared_ptr<const void>> *find(const void *kernel, int chunk) const {
+        for (const Entry &e : entries)
+            if (e.kernel == kernel && e.chunk == chunk) return &e.blocks;
+        return nullptr;
+    }
+};
+
 // Splits tensors [0, n) into parameter blocks of tiles of `chunk` elements and
 // launches `kernel` once per block.
-// fill(p, ptrs) writes tensor p's pointers.
+// fill(p, ptrs) writes tensor p's pointers.  With a cache, the blocks are taken from it, or
+// built once and kept there.
 template <int NP, typename Kernel, typename Fill>
 int launch_streaming(Kernel kernel, int n, const int64_t *numels, int chunk, int threads,
                      int smem, const Scalars &sc, int grid_override, cudaStream_t stream,
-                     Fill fill) {
+                     Fill fill, TableCache *cache = nullptr) {
     using T = Table<NP>;
     const int grid_cap = resident_ctas((const void *)kernel, threads, smem);
     if (grid_cap <= 0) {
         g_last_cuda = (int)cudaGetLastError();
         return TULA_ERR_CUDA;
     }
-    std::vector<std::unique_ptr<T>> tabs;
-    long long c_global = 0;
-    int p = 0;
-    while (p < n) {
-        std::unique_ptr<T> tab(new T);
-        std::memset(tab.get(), 0, sizeof(T));
-        tab->t0 = p;
-        tab->c0 = (int)c_global;
-        tab->chunk = chunk;
-        int cnt = 0, nc = 0;
-        while (p < n && cnt < T::kMaxT) {
-            tab->numel[cnt] = numels[p];
-            tab->cstart[cnt] = nc;
-            fill(p, tab->ptr[cnt]);
-            nc += (int)tiles_of(numels[p], chunk);
-            ++cnt;
-            ++p;
+    const std::vector<std::shared_ptr<const void>> *blocks =
+        cache ? cache->find((const void *)kernel, chunk) : nullptr;
+    std::vector<std::shared_ptr<const void>> built;
+    if (!blocks) {
+        try {
+            long long c_global = 0;
+            int p = 0;
+            while (p < n) {
+                std::shared_ptr<T> tab = std::make_shared<T>();
+                std::memset(tab.get(), 0, sizeof(T));
+                tab->t0 = p;
+                tab->c0 = (int)c_global;
+                tab->chunk = chunk;
+                tab->first = p == 0 ? 1 : 0;
+                int cnt = 0, nc = 0;
+                while (p < n && cnt < T::kMaxT) {
+                    tab->numel[cnt] = numels[p];
+                    tab->cstart[cnt] = nc;
+                    fill(p, tab->ptr[cnt]);
+                    nc += (int)tiles_of(numels[p], chunk);
+                    ++cnt;
+                    ++p;
+                }
+                tab->n = cnt;
+                tab->nc = nc;
+                tab->cstart[cnt] = nc;
+                c_global += nc;
+                built.push_back(std::move(tab));
+            }
+            if (cache) {
+                cache->entries.push_back({(const void *)kernel, chunk, std::move(built)});
+                blocks = &cache->entries.back().blocks;
+            }
+        } catch (const std::bad_alloc &) {
+            return TULA_ERR_NO_MEMORY;
         }
-        tab->n = cnt;
-        tab->nc = nc;
-        tab->cstart[cnt] = nc;
-        c_global += nc;
-        tabs.push_back(std::move(tab));
+        if (!blocks) blocks = &built;
     }
-    tabs.front()->first = 1;
-    for (const auto &tab : tabs) {
+    for (const auto &b : *blocks) {
+        const T &tab = *static_cast<const T *>(b.get());
         int grid = grid_override > 0 ? grid_override : grid_cap;
-        grid = std::max(1, std::min(grid, tab->nc));
-        const int rc = launch_pdl(kernel, grid, threads, smem, stream, *tab, sc);
+        grid = std::max(1, std::min(grid, tab.nc));
+        const int rc = launch_pdl(kernel, grid, threads, smem, stream, tab, sc);
         if (rc) return rc;
     }
     return TULA_OK;
@@ -2035,11 +2068,11 @@ void record(void *ev, cudaStream_t s) {
 // Pass 1 (+ its finish) dispatched over the compile-time replica count.
 template <int KT, bool WM, bool RW, bool SS, bool PR, typename Fill>
 int run_reduce_k(int K, int n, const int64_t *numels, const Scalars &sc, int grid, cudaStream_t s,
-                 Fill fill, void *mid_event, bool finish) {
+                 Fill fill, void *mid_event, bool finish, TableCache *cache) {
     const int chunk = chunk1(K, RW, SS);
     int rc = launch_streaming<P1<KT>::NP>(k_reduce<KT, WM, RW, SS, PR>, n, numels, chunk,
                                           Ring1::kThreads, Ring1::kSmemBytes, sc,
-                                          grid, s, fill);
+                                          grid, s, fill, cache);
     if (rc) return rc;
     record(mid_event, s);
     return finish ? launch_finish<kAcc>(n, sc, s) : TULA_OK;
@@ -2047,14 +2080,15 @@ int run_reduce_k(int K, int n, const int64_t *numels, const Scalars &sc, int gri
 
 template <bool WM, bool RW, bool SS, bool PR, typename Fill>
 int run_reduce(int K, int n, const int64_t *numels, const Scalars &sc, int grid, cudaStream_t s,
-               Fill fill, void *mid_event = nullptr, bool finish = true) {
+               Fill fill, void *mid_event = nullptr, bool finish = true,
+               TableCache *cache = nullptr) {
     switch (K) {
-    case 1: return run_reduce_k<1, false, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish);
-    case 2: return run_reduce_k<2, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish);
-    case 4: return run_reduce_k<4, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish);
-    case 8: return run_reduce_k<8, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish);
-    case 16: return run_reduce_k<16, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish);
-    default: return run_reduce_k<0, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish);
+    case 1: return run_reduce_k<1, false, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish, cache);
+    case 2: return run_reduce_k<2, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish, cache);
+    case 4: return run_reduce_k<4, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish, cache);
+    case 8: return run_reduce_k<8, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish, cache);
+    case 16: return run_reduce_k<16, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish, cache);
+    default: return run_reduce_k<0, WM, RW, SS, PR>(K, n, numels, sc, grid, s, fill, mid_event, finish, cache);
     }
 }
 
@@ -2157,12 +2191,10 @@ namespace {
 
 // Every host-side check of a step's arguments except the workspace: TULA_OK or the status
 // tula_ags_step returns.  Nothing is enqueued before it passes.
-int check_step_args(float *const *param_ptrs, float *const *grad_ptrs, float *const *mom_ptrs,
-                    const int64_t *numels, int n_tensors, float momentum,
-                    const tula_ags_hparams *hp, Plan *pl) {
-    if (!hp || !param_ptrs || !grad_ptrs || !valid_numels(numels, n_tensors, hp->K, pl))
-        return TULA_ERR_ARG;
-    const int K = hp->K, n = n_tensors;
+// The options of a step (hp apart from its workspace, and the momentum) against the buffers the
+// step has: momentum buffers (has_mom) and per-element gradscales (has_se).
+int check_step_options(const tula_ags_hparams *hp, float momentum, bool has_mom, bool has_se) {
+    if (!hp || hp->K < 1 || hp->K > TULA_MAX_K) return TULA_ERR_ARG;
     if (hp->rule < TULA_RULE_AGS || hp->rule > TULA_RULE_STATIC) return TULA_ERR_ARG;
     if (hp->granularity != TULA_SCALE_PER_TENSOR && hp->granularity != TULA_SCALE_PER_ELEMENT)
         return TULA_ERR_ARG;
@@ -2171,23 +2203,41 @@ int check_step_args(float *const *param_ptrs, float *const *grad_ptrs, float *co
     if (!hp->state) return TULA_ERR_ARG;
     const bool per_elem = hp->rule == TULA_RULE_AGS && hp->granularity == TULA_SCALE_PER_ELEMENT;
     if (hp->rule == TULA_RULE_AGS && !per_elem && !hp->scale) return TULA_ERR_ARG;
-    if (per_elem && !hp->scale_elem) return TULA_ERR_ARG;
-    if (!mom_ptrs && momentum != 0.0f) return TULA_ERR_ARG;
+    if (per_elem && !has_se) return TULA_ERR_ARG;
+    if (!has_mom && momentum != 0.0f) return TULA_ERR_ARG;
     if (hp->refresh_scale) {
-        if (K == 1 || !hp->scale) return TULA_ERR_ARG;
+        if (hp->K == 1 || !hp->scale) return TULA_ERR_ARG;
         if (hp->granularity != TULA_SCALE_PER_TENSOR) return TULA_ERR_UNSUPPORTED;
     }
+    return TULA_OK;
+}
+
+// The tensors of a step: their sizes, and every pointer of a non-empty tensor non-NULL and
+// 4-byte aligned (scale_elem: the per-element gradscales, or NULL when the step has none).
+int check_step_tensors(float *const *param_ptrs, float *const *grad_ptrs, float *const *mom_ptrs,
+                       float *const *scale_elem, const int64_t *numels, int n, int K, Plan *pl) {
+    if (!param_ptrs || !grad_ptrs || !valid_numels(numels, n, K, pl)) return TULA_ERR_ARG;
     for (int p = 0; p < n; ++p) {
         if (numels[p] == 0) continue;
         if (!param_ptrs[p] || !aligned4(param_ptrs[p])) return TULA_ERR_ARG;
         if (mom_ptrs && (!mom_ptrs[p] || !aligned4(mom_ptrs[p]))) return TULA_ERR_ARG;
-        if (per_elem && (!hp->scale_elem[p] || !aligned4(hp->scale_elem[p]))) return TULA_ERR_ARG;
+        if (scale_elem && (!scale_elem[p] || !aligned4(scale_elem[p]))) return TULA_ERR_ARG;
         for (int k = 0; k < K; ++k) {
             const float *g = grad_ptrs[(size_t)k * n + p];
             if (!g || !aligned4(g)) return TULA_ERR_ARG;
         }
     }
     return TULA_OK;
+}
+
+int check_step_args(float *const *param_ptrs, float *const *grad_ptrs, float *const *mom_ptrs,
+                    const int64_t *numels, int n_tensors, float momentum,
+                    const tula_ags_hparams *hp, Plan *pl) {
+    int rc = check_step_options(hp, momentum, mom_ptrs != nullptr, hp && hp->scale_elem);
+    if (rc) return rc;
+    const bool per_elem = hp->rule == TULA_RULE_AGS && hp->granularity == TULA_SCALE_PER_ELEMENT;
+    return check_step_tensors(param_ptrs, grad_ptrs, mom_ptrs, per_elem ? hp->scale_elem : nullptr,
+                              numels, n_tensors, hp->K, pl);
 }
 
 // Which part of a step run_step launches: all of it, or one half of a sharded step (pass 1 up to
@@ -2200,7 +2250,7 @@ int run_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mo
              const int64_t *numels, int n, float lr, float momentum, float weight_decay,
              const tula_ags_hparams *hp, void *ws, const Plan &pl, void *stream,
              StepPart part = kPartWhole, unsigned long long *share_out = nullptr,
-             const unsigned long long *g2_in = nullptr) {
+             const unsigned long long *g2_in = nullptr, TableCache *cache = nullptr) {
     const int K = hp->K;
     const bool per_elem = hp->rule == TULA_RULE_AGS && hp->granularity == TULA_SCALE_PER_ELEMENT;
     int rc = TULA_OK;
@@ -2238,13 +2288,13 @@ int run_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mo
         // Norms feeding a coefficient (LARS, UpdateGradScale) are taken precisely.
         if (lars)
             rc = run_reduce<true, true, false, true>(K, n, numels, sc, hp->grid_ctas, s, fill1,
-                                                     hp->trace_events[1], fin);
+                                                     hp->trace_events[1], fin, cache);
         else if (hp->refresh_scale)
             rc = run_reduce<true, false, false, true>(K, n, numels, sc, hp->grid_ctas, s, fill1,
-                                                      hp->trace_events[1], fin);
+                                                      hp->trace_events[1], fin, cache);
         else
             rc = run_reduce<true, false, false, false>(K, n, numels, sc, hp->grid_ctas, s, fill1,
-                                                       hp->trace_events[1], fin);
+                                                       hp->trace_events[1], fin, cache);
         if (rc == TULA_OK && part == kPartReduce)
             return launch_pdl(k_share, 1, 32, 0, s, sc, share_out);
     }
@@ -2265,7 +2315,7 @@ int run_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mo
     sc.mode = kModeUpdate;
 #define TULA_UPD(HM, PE, SW)                                                                \
     launch_streaming<kNP2>(k_update<HM, PE, SW>, n, numels, c2, Ring2::kThreads,             \
-                           Ring2::kSmemBytes, sc, hp->grid_ctas, s, fill2)
+                           Ring2::kSmemBytes, sc, hp->grid_ctas, s, fill2, cache)
     if (hm) {
         if (per_elem) rc = sw ? TULA_UPD(true, true, true) : TULA_UPD(true, true, false);
         else rc = sw ? TULA_UPD(true, false, true) : TULA_UPD(true, false, false);
@@ -2284,6 +2334,16 @@ int run_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mo
 
 }  // namespace
 
+// A plan (tula_ags_plan_create): the step's sizes and pointer arrays, checked once, on one
+// device, and the launch tables built from them by the first step of each kernel variant.
+struct tula_ags_plan {
+    int n = 0, K = 0, device = 0;
+    Plan tiles;
+    std::vector<int64_t> numels;
+    std::vector<float *> params, grads, moms, scale_elem;
+    TableCache tables;
+};
+
 extern "C" {
 
 int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *const *mom_ptrs,
@@ -2296,6 +2356,68 @@ int tula_ags_step(float *const *param_ptrs, float *const *grad_ptrs, float *cons
     if (rc) return rc;
     return run_step(param_ptrs, grad_ptrs, mom_ptrs, numels, n_tensors, lr, momentum,
                     weight_decay, hp, hp->workspace, pl, stream);
+}
+
+int tula_ags_plan_create(float *const *param_ptrs, float *const *grad_ptrs,
+                         float *const *mom_ptrs, const int64_t *numels, int n_tensors,
+                         const tula_ags_hparams *hp, tula_ags_plan **plan_out) {
+    if (!plan_out) return TULA_ERR_ARG;
+    *plan_out = nullptr;
+    if (!hp || hp->K < 1 || hp->K > TULA_MAX_K) return TULA_ERR_ARG;
+    Plan pl;
+    int rc = check_step_tensors(param_ptrs, grad_ptrs, mom_ptrs, hp->scale_elem, numels,
+                                n_tensors, hp->K, &pl);
+    if (rc) return rc;
+    int dev = 0;
+    const cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) {
+        g_last_cuda = (int)e;
+        return TULA_ERR_CUDA;
+    }
+    try {
+        std::unique_ptr<tula_ags_plan> P(new tula_ags_plan);
+        const size_t n = (size_t)n_tensors, K = (size_t)hp->K;
+        P->n = n_tensors;
+        P->K = hp->K;
+        P->device = dev;
+        P->tiles = pl;
+        P->numels.assign(numels, numels + n);
+        P->params.assign(param_ptrs, param_ptrs + n);
+        P->grads.assign(grad_ptrs, grad_ptrs + K * n);
+        if (mom_ptrs) P->moms.assign(mom_ptrs, mom_ptrs + n);
+        if (hp->scale_elem) P->scale_elem.assign(hp->scale_elem, hp->scale_elem + n);
+        *plan_out = P.release();
+    } catch (const std::bad_alloc &) {
+        return TULA_ERR_NO_MEMORY;
+    }
+    return TULA_OK;
+}
+
+int tula_ags_plan_step(tula_ags_plan *plan, float lr, float momentum, float weight_decay,
+                       const tula_ags_hparams *hp, void *stream) {
+    if (!plan || !hp || hp->K != plan->K) return TULA_ERR_ARG;
+    int rc = check_step_options(hp, momentum, !plan->moms.empty(), !plan->scale_elem.empty());
+    if (rc) return rc;
+    rc = check_ws(hp->workspace, hp->workspace_bytes, plan->n, plan->tiles);
+    if (rc) return rc;
+    int dev = 0;
+    const cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) {
+        g_last_cuda = (int)e;
+        return TULA_ERR_CUDA;
+    }
+    if (dev != plan->device) return TULA_ERR_ARG;
+    tula_ags_hparams h = *hp;
+    h.scale_elem = plan->scale_elem.empty() ? nullptr : plan->scale_elem.data();
+    return run_step(plan->params.data(), plan->grads.data(),
+                    plan->moms.empty() ? nullptr : plan->moms.data(), plan->numels.data(),
+                    plan->n, lr, momentum, weight_decay, &h, h.workspace, plan->tiles, stream,
+                    kPartWhole, nullptr, nullptr, &plan->tables);
+}
+
+int tula_ags_plan_destroy(tula_ags_plan *plan) {
+    delete plan;
+    return TULA_OK;
 }
 
 int tula_ags_shard_reduce(float *const *param_ptrs, float *const *grad_ptrs,
@@ -2400,7 +2522,7 @@ int tula_ags_update_scale(const float *const *g_small, const float *const *g_lar
         dst[2] = g_small[p];
     };
     return run_reduce_k<1, false, false, true, true>(1, n, numels, sc, hp->grid_ctas, s, fill,
-                                                     nullptr, true);
+                                                     nullptr, true, nullptr);
 }
 
 const char *tula_ags_error_string(int code) {
@@ -2413,6 +2535,7 @@ const char *tula_ags_error_string(int code) {
     case TULA_ERR_SCRATCH_LIMIT:
         return "tensor list needs more than the library's static scratch "
                "(TULA_STATIC_SCRATCH_BYTES); use tula_ags_step with a workspace";
+    case TULA_ERR_NO_MEMORY: return "host memory allocation failed";
     default: return "unknown status";
     }
 }

@@ -19,7 +19,7 @@ from .build import HEADER, LIB
 c_int, c_float, c_void_p, c_size_t = ctypes.c_int, ctypes.c_float, ctypes.c_void_p, ctypes.c_size_t
 
 TULA_OK, TULA_ERR_ARG, TULA_ERR_WORKSPACE, TULA_ERR_CUDA, TULA_ERR_UNSUPPORTED = 0, -1, -2, -3, -4
-TULA_ERR_SCRATCH_LIMIT = -5
+TULA_ERR_SCRATCH_LIMIT, TULA_ERR_NO_MEMORY = -5, -6
 TULA_STATIC_SCRATCH_BYTES = 16 << 20
 TULA_MAX_K = 16
 TULA_RULE_AGS, TULA_RULE_NONE, TULA_RULE_LARS, TULA_RULE_STATIC = 0, 1, 2, 3
@@ -96,11 +96,15 @@ def lib() -> ctypes.CDLL:
     L.tula_ags_shard_update.argtypes = [pp, pp, pp, i64p, c_int, c_float, c_float, c_float, hpp,
                                         c_void_p, c_void_p]
     L.tula_ags_static_scratch_check_wait_timeout.argtypes = [c_void_p]
+    L.tula_ags_plan_create.argtypes = [pp, pp, pp, i64p, c_int, hpp, ctypes.POINTER(c_void_p)]
+    L.tula_ags_plan_step.argtypes = [c_void_p, c_float, c_float, c_float, hpp, c_void_p]
+    L.tula_ags_plan_destroy.argtypes = [c_void_p]
     for name in ("tula_ags_workspace_size", "tula_ags_step", "tula_layer_stats",
                  "tula_ags_update_scale", "tula_ags_plan_chunks", "tula_ags_step_static_scratch",
                  "tula_ags_workspace_error", "tula_ags_check_wait_timeout",
                  "tula_ags_static_scratch_error", "tula_ags_static_scratch_check_wait_timeout",
-                 "tula_ags_shard_reduce", "tula_ags_shard_update"):
+                 "tula_ags_shard_reduce", "tula_ags_shard_update", "tula_ags_plan_create",
+                 "tula_ags_plan_step", "tula_ags_plan_destroy"):
         getattr(L, name).restype = c_int
     _lib = L
     return L
@@ -246,6 +250,29 @@ def tula_ags_step(params, grads, moms, lr, momentum, weight_decay, hp: tula_ags_
     _check(rc, "tula_ags_step")
 
 
+def tula_ags_plan_create(params, grads, moms, hp: tula_ags_hparams) -> c_void_p:
+    """A plan over fixed tensors (hp.K, hp.scale_elem read); the tensors must outlive it."""
+    flat = _replica_list(params, grads, hp, "tula_ags_plan_create", moms)
+    plan = c_void_p()
+    rc = lib().tula_ags_plan_create(_tensor_ptrs(params), _tensor_ptrs(flat),
+                                    _tensor_ptrs(moms) if moms is not None else None,
+                                    _numels(params), len(params), ctypes.byref(hp),
+                                    ctypes.byref(plan))
+    _check(rc, "tula_ags_plan_create")
+    return plan
+
+
+def tula_ags_plan_step(plan: c_void_p, lr, momentum, weight_decay, hp: tula_ags_hparams,
+                       stream=None) -> None:
+    rc = lib().tula_ags_plan_step(plan, lr, momentum, weight_decay, ctypes.byref(hp),
+                                  _stream_ptr(stream))
+    _check(rc, "tula_ags_plan_step")
+
+
+def tula_ags_plan_destroy(plan: c_void_p) -> None:
+    _check(lib().tula_ags_plan_destroy(plan), "tula_ags_plan_destroy")
+
+
 def tula_ags_step_static_scratch(params, grads, moms, lr, momentum, weight_decay,
                                  hp: tula_ags_hparams, stream=None) -> None:
     """tula_ags_step for callers that cannot allocate device memory: the step's scratch is
@@ -305,12 +332,14 @@ class AGSOptimizerStep:
     model so that each step is a single C call.
 
     params, moms: n tensors; grads: K lists of n tensors (replica k of tensor p).
+    plan: step through a tula_ags_plan (sizes and pointers checked once, launch tables
+    reused) rather than through tula_ags_step; the results are the same bit for bit.
     """
 
     def __init__(self, params, grads, moms=None, *, rule=TULA_RULE_AGS,
                  granularity=TULA_SCALE_PER_TENSOR, delta=0.5, eps=1e-8, s_max=None,
                  static_s=1.0, lars_trust=1.0, force_branch=TULA_BRANCH_AUTO, scale=None,
-                 scale_elem=None, stats=True, grid_ctas=0):
+                 scale_elem=None, stats=True, grid_ctas=0, plan=True):
         self.params = list(params)
         self.grads = [list(r) for r in grads]
         self.moms = list(moms) if moms is not None else None
@@ -353,6 +382,14 @@ class AGSOptimizerStep:
         self._g = _tensor_ptrs(flat)
         self._m = _tensor_ptrs(self.moms) if self.moms is not None else None
         self._numels = _numels(self.params)
+        self._plan = None
+        if plan:
+            handle = c_void_p()
+            _check(lib().tula_ags_plan_create(self._p, self._g, self._m, self._numels, self.n,
+                                              ctypes.byref(self.hp), ctypes.byref(handle)),
+                   "tula_ags_plan_create")
+            self._plan = handle
+            self._destroy = lib().tula_ags_plan_destroy  # kept for __del__ at shutdown
         # The zero fills above ran on the current stream; steps may be issued on any other
         # (torch's side streams do not wait for it), so finish them before the first step.
         torch.cuda.synchronize(dev)
@@ -371,9 +408,20 @@ class AGSOptimizerStep:
 
     def step(self, lr, momentum, weight_decay, refresh_scale=False, stream=None) -> None:
         self.hp.refresh_scale = 1 if refresh_scale else 0
+        if self._plan is not None:
+            rc = lib().tula_ags_plan_step(self._plan, lr, momentum, weight_decay,
+                                          ctypes.byref(self.hp), _stream_ptr(stream))
+            _check(rc, "tula_ags_plan_step")
+            return
         rc = lib().tula_ags_step(self._p, self._g, self._m, self._numels, self.n, lr, momentum,
                                  weight_decay, ctypes.byref(self.hp), _stream_ptr(stream))
         _check(rc, "tula_ags_step")
+
+    def __del__(self):
+        plan = getattr(self, "_plan", None)
+        if plan is not None:
+            self._plan = None
+            self._destroy(plan)
 
     __call__ = step
 

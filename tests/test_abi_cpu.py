@@ -190,3 +190,43 @@ def test_sharded_step_argument_errors(lib):
     hp.state = 0
     assert lib.tula_ags_shard_reduce(ptrs, ptrs, ptrs, numels, 2, 0.9, ctypes.byref(hp),
                                      0x50000, None) == T.TULA_ERR_ARG
+
+
+def test_plan_argument_errors_come_before_any_cuda_call(lib):
+    """tula_ags_plan_create checks the sizes and every pointer before it asks CUDA for the
+    current device, and tula_ags_plan_step refuses a NULL plan or hp; no GPU is needed to see
+    TULA_ERR_ARG, and *plan_out stays NULL on every error."""
+    P = ctypes.c_void_p
+    ptrs = (P * 4)(*[0x100000 * (i + 1) for i in range(4)])
+    numels = (ctypes.c_int64 * 2)(5, 7)
+    hp = T.tula_ags_default_hparams(2)
+    out = P(0x1234)
+    create = lib.tula_ags_plan_create
+    assert create(ptrs, ptrs, ptrs, numels, 2, ctypes.byref(hp), None) == T.TULA_ERR_ARG
+    assert create(ptrs, ptrs, ptrs, numels, 2, None, ctypes.byref(out)) == T.TULA_ERR_ARG
+    assert out.value is None
+    bad = (P * 4)(0x100000, 0x100002, 0x100000, 0x100000)     # misaligned second gradient
+    assert create(ptrs, bad, ptrs, numels, 2, ctypes.byref(hp), ctypes.byref(out)) == T.TULA_ERR_ARG
+    nul = (P * 4)(0x100000, None, 0x100000, 0x100000)          # a missing momentum buffer
+    assert create(ptrs, ptrs, nul, numels, 2, ctypes.byref(hp), ctypes.byref(out)) == T.TULA_ERR_ARG
+    hp.K = 0
+    assert create(ptrs, ptrs, ptrs, numels, 2, ctypes.byref(hp), ctypes.byref(out)) == T.TULA_ERR_ARG
+    hp.K = 2
+    neg = (ctypes.c_int64 * 2)(5, -1)
+    assert create(ptrs, ptrs, ptrs, neg, 2, ctypes.byref(hp), ctypes.byref(out)) == T.TULA_ERR_ARG
+    assert out.value is None
+    assert lib.tula_ags_plan_step(None, 0.1, 0.9, 0.0, ctypes.byref(hp), None) == T.TULA_ERR_ARG
+    assert lib.tula_ags_plan_destroy(None) == T.TULA_OK
+    assert "allocation" in T.tula_ags_error_string(T.TULA_ERR_NO_MEMORY)
+
+
+def test_plan_binding_checks_replica_lists(lib):
+    """The wrapper refuses replica and momentum lists that do not match hp.K and the tensor
+    count, before the C call (which reads K * n gradient pointers)."""
+    import torch
+    params = [torch.zeros(4), torch.zeros(4)]
+    hp = T.tula_ags_default_hparams(2)
+    with pytest.raises(ValueError, match="replica"):
+        T.tula_ags_plan_create(params, [params], params, hp)
+    with pytest.raises(ValueError, match="momentum"):
+        T.tula_ags_plan_create(params, [params, params], params[:1], hp)

@@ -664,3 +664,85 @@ def test_sharded_step_equals_the_whole_step(name, rule):
         for x, y in ((a.w_flat, b.w_flat), (a.m_flat, b.m_flat), (a.g_flats[0], b.g_flats[0])):
             assert torch.equal(x, y), where
     assert [int(v) for v in (whole.state[1].item(),)] == [4]
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("case", ["ragged_k4", "many_k2", "no_momentum"])
+def test_plan_steps_equal_direct_steps(case):
+    """A plan (tula_ags_plan_create) checks the tensors once and keeps the launch tables of each
+    kernel variant from its first use.  Switching rule, granularity, refresh, branch and grid
+    between steps -- each a variant the plan builds once and then reuses -- must give bit for bit
+    the w, m, mean, step record, statistics and gradscale of tula_ags_step with the same
+    arguments.  The plan also refuses what it was not created with."""
+    if case == "many_k2":
+        rng = np.random.default_rng(171)
+        ps = W.ParamSet("many")
+        for n in rng.integers(1, 3000, size=800):   # several parameter blocks per pass
+            ps.add((int(n),), W.KIND_NORMAL)
+        K = 2
+    else:
+        ps, K = _ragged_pset(K=4), 4
+    mom = case != "no_momentum"
+    wl = W.workload("stress_k4", seed=171, factor_range=(0.1, 10.0), zero_patterns=False)
+    bufs = [W.allocate(wl, "cuda", K=K, pset=ps, with_momentum=mom) for _ in range(2)]
+    for b in bufs:
+        W.fill_state(b, wl)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(172)
+    se0 = [torch.rand(t.numel(), generator=gen, device="cuda") * 2 for t in bufs[0].w]
+    se = [se0, [x.clone() for x in se0]]
+    kw = dict(s_max=2.0, lars_trust=0.01, static_s=0.5)
+    st = [T.AGSOptimizerStep(b.w, b.g, b.m if mom else None, scale_elem=se[i], plan=(i == 0), **kw)
+          for i, b in enumerate(bufs)]
+    assert st[0]._plan is not None and st[1]._plan is None
+    mu = 0.9 if mom else 0.0
+    schedule = [
+        (1, 1.0, dict(refresh=True)),
+        (1, 1.0, dict()),                                    # Delta = 0: scaled
+        (2, 2.0, dict(grid=7)),                              # Delta = 3: unscaled
+        (2, 1.0, dict(rule=T.TULA_RULE_LARS)),
+        (3, 1.0, dict(gran=T.TULA_SCALE_PER_ELEMENT, force=T.TULA_BRANCH_SCALED)),
+        (3, 1.0, dict(gran=T.TULA_SCALE_PER_ELEMENT)),
+        (4, 1.0, dict(rule=T.TULA_RULE_STATIC, force=T.TULA_BRANCH_SCALED, grid=333)),
+        (4, 1.0, dict(rule=T.TULA_RULE_NONE)),
+        (5, 1.0, dict(refresh=True)),
+        (5, 1.0, dict()),
+    ]
+    for i, (seed_step, mult, o) in enumerate(schedule):
+        for b, s in zip(bufs, st):
+            W.fill_grads(b, wl, step=seed_step, multiplier=mult)
+            s.hp.rule = o.get("rule", T.TULA_RULE_AGS)
+            s.hp.granularity = o.get("gran", T.TULA_SCALE_PER_TENSOR)
+            s.hp.force_branch = o.get("force", T.TULA_BRANCH_AUTO)
+            s.hp.grid_ctas = o.get("grid", 0)
+            s.step(wl.lr, mu, wl.weight_decay, refresh_scale=o.get("refresh", False))
+        torch.cuda.synchronize()
+        where = f"{case} step {i + 1} {o}"
+        a, b = bufs
+        assert torch.equal(a.w_flat, b.w_flat), where + " w"
+        assert torch.equal(a.g_flats[0], b.g_flats[0]), where + " mean"
+        if mom:
+            assert torch.equal(a.m_flat, b.m_flat), where + " m"
+        for name in ("state", "stats", "scale"):   # bit patterns: the statistics hold NaN
+            x, y = getattr(st[0], name), getattr(st[1], name)
+            it = torch.int64 if x.dtype == torch.float64 else torch.int32
+            assert torch.equal(x.view(it), y.view(it)), where + " " + name
+    assert st[0].state[1].item() == len(schedule)
+    p = st[0]
+    p.hp.rule, p.hp.granularity, p.hp.force_branch, p.hp.grid_ctas = T.TULA_RULE_AGS, 0, 0, 0
+    p.hp.K = K + 1                                             # not the plan's K
+    with pytest.raises(T.TulaError) as e:
+        p.step(0.1, mu, 0.0)
+    assert e.value.code == T.TULA_ERR_ARG
+    p.hp.K = K
+    if not mom:
+        with pytest.raises(T.TulaError) as e:                  # no momentum buffers in the plan
+            p.step(0.1, 0.9, 0.0)
+        assert e.value.code == T.TULA_ERR_ARG
+    bare = T.AGSOptimizerStep(bufs[0].w, bufs[0].g, bufs[0].m if mom else None, **kw)
+    bare.hp.granularity = T.TULA_SCALE_PER_ELEMENT             # created without scale_elem
+    with pytest.raises(T.TulaError) as e:
+        bare.step(0.1, mu, 0.0)
+    assert e.value.code == T.TULA_ERR_ARG
+    torch.cuda.synchronize()
+    assert p.error() == 0
