@@ -746,3 +746,52 @@ def test_plan_steps_equal_direct_steps(case):
     assert e.value.code == T.TULA_ERR_ARG
     torch.cuda.synchronize()
     assert p.error() == 0
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("delta", [0.5, 0.1, 0.3, 1.0, 0.25, 2.0])
+def test_branch_at_the_rounding_boundary_of_delta(delta):
+    """Algorithm 1's branch where the rounded Delta of Eq. 5 meets delta.  |G|^2 is fixed by
+    integer gradients (K = 1, so the sum is exact); the previous |G|^2 is planted in the step
+    record on both sides of G2 and stepped one ulp at a time across the point where
+    fl(|fl(G2 - G2_prev)| / G2_prev) reaches delta.  Delta (bit for bit) and the branch must be
+    those of the fp64 formula for every candidate, both branches must occur, and a first step
+    (no previous norm) is unscaled."""
+    n = 4099
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(181)
+    g = torch.randint(-9, 10, (n,), generator=gen, device="cuda").float()
+    g2 = float(np.sum(g.cpu().numpy().astype(np.float64) ** 2))   # exact: integers < 2^53
+    w = torch.zeros(n, device="cuda")
+    m = torch.zeros(n, device="cuda")
+    st = T.AGSOptimizerStep([w], [[g]], [m], s_max=1.0, delta=delta, stats=False)
+    d32 = float(np.float32(delta))
+    seen = set()
+    for sign in (1.0, -1.0):
+        if sign < 0 and d32 >= 1.0:
+            continue                              # G2_prev would have to be negative
+        centre = g2 / (1.0 + sign * d32)          # |g2 - g2p| / g2p = delta near here
+        cands = [centre]
+        for direction in (np.inf, -np.inf):
+            x = centre
+            for _ in range(6):
+                x = float(np.nextafter(x, direction))
+                cands.append(x)
+        for g2p in cands:
+            st.state.copy_(torch.tensor([g2p, 3.0, 0.0, 0.0], dtype=torch.float64))
+            st.step(0.0, 0.0, 0.0)
+            torch.cuda.synchronize()
+            dv = abs((np.float64(g2) - np.float64(g2p)) / np.float64(g2p))
+            want = int(dv < np.float64(d32))
+            got = st.state.cpu().numpy()
+            assert got[0] == g2 and got[1] == 4.0, g2p
+            assert got[2] == dv, (g2p, got[2], dv)
+            assert int(got[3]) == want, (delta, g2p, dv)
+            seen.add(want)
+    assert seen == {0, 1}
+    st.state.zero_()                              # a first step: Delta = +inf, unscaled
+    st.step(0.0, 0.0, 0.0)
+    torch.cuda.synchronize()
+    got = st.state.cpu().numpy()
+    assert np.isinf(got[2]) and got[3] == 0.0
+    assert st.error() == 0
