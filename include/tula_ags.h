@@ -334,10 +334,11 @@ uint64_t tula_ags_launch_count(void);
 
 /*
  * Elements per tile (work item) of a pass that streams `streams` tensors through shared memory:
- * pass 1, the reduction (K replicas [+ w] [+ g_small]; one tile of every stream fills a 36 KB
- * stage), or pass 2, the update (gbar, w [+ m] [+ per-element scale]; a 24 KB stage).  A multiple
- * of 128; TULA_ERR_ARG for another pass or when streams is outside [1, TULA_MAX_K + 2] (pass 1)
- * or [1, 4] (pass 2).
+ * pass 1, the reduction (K replicas [+ g_small]; one tile of every stream fills a 36 KB stage),
+ * pass 2, the update (gbar, w [+ m] [+ per-element scale]; a 24 KB stage), or pass 3, the
+ * reduction when it also reads w (K replicas + w: LARS steps and tula_layer_stats; a 45 KB
+ * stage).  A multiple of 128; TULA_ERR_ARG for another pass or when streams is outside
+ * [1, TULA_MAX_K + 2] (passes 1 and 3) or [1, 4] (pass 2).
  */
 int tula_ags_chunk_elems(int pass, int streams);
 

@@ -82,6 +82,13 @@ struct Ring {
 // the default ones add their tile sums into the accumulators at the end of each batch; with
 // three warps the reduction ran 0.8 % slower alone (the same step time).
 using Ring1 = Ring<36, 6, 6>;
+// Pass 1 when it also reads w (LARS, tula_layer_stats) streams through five 45 KB stages with
+// five consumers: the larger tiles (1280 elements for K = 8 and w) make every bulk copy 5 KB
+// instead of 4 KB, and the LARS step ran 2.5 % faster (ResNet-50, 248.1 -> 241.9 us); without
+// w (8 streams) the same ring measured 0.5 % slower.
+using Ring1W = Ring<45, 5, 5>;
+template <bool RW>
+using Ring1Of = std::conditional_t<RW, Ring1W, Ring1>;
 // Pass 2 does ~11 flops per element over 3-4 streams: with three consumer warps they, not HBM,
 // set its pace, so it runs four.
 using Ring2 = Ring<24, 8, 4>;
@@ -953,7 +960,7 @@ __device__ __forceinline__ void reduce_tile(uint32_t stage, int chunk, const flo
     float fg = 0.f, fs = 0.f, fw = 0.f;   // fp32 sums (not PR)
 
     if constexpr (KT > 0) {
-        constexpr int CH = Ring1::tile_elems(KT + (RW ? 1 : 0) + (SS ? 1 : 0));
+        constexpr int CH = Ring1Of<RW>::tile_elems(KT + (RW ? 1 : 0) + (SS ? 1 : 0));
         constexpr int COLS = CH / 128;  // float4 columns per lane of a full tile
         if (nv == CH / 4) {
             // Full tile: every lane has COLS columns; all loads of a column issue together.
@@ -1126,7 +1133,7 @@ __device__ __noinline__ void add_tile_now(const Scalars &sc, int tg, const float
 }
 
 template <int KT, bool WM, bool RW, bool SS, bool PR>
-__global__ void __launch_bounds__(Ring1::kThreads, 1)
+__global__ void __launch_bounds__(Ring1Of<RW>::kThreads, 1)
     k_reduce(const __grid_constant__ Table<P1<KT>::NP> tab, const __grid_constant__ Scalars sc) {
     constexpr int KS = P1<KT>::KS;
     constexpr int NSMAX = KS + 2;
@@ -1146,7 +1153,7 @@ __global__ void __launch_bounds__(Ring1::kThreads, 1)
     if (!early) grid_wait();
     uint64_t *full, *empty;
     int *stage_tile;
-    using R1 = Ring1;
+    using R1 = Ring1Of<RW>;
     ring_setup<R1>(smem, full, empty, stage_tile);
     const int js = static_tiles(tab.nc);
     const uint32_t ring = smem_addr(smem);
@@ -1818,10 +1825,12 @@ inline int replica_slot(int K) {
 
 // Tile sizes: the smallest a pass can use for K replicas sizes the workspace.
 inline int chunk1(int K, bool rw, bool ss) {
-    return Ring1::tile_elems(K + (rw ? 1 : 0) + (ss ? 1 : 0));
+    const int streams = K + (rw ? 1 : 0) + (ss ? 1 : 0);
+    return rw ? Ring1W::tile_elems(streams) : Ring1::tile_elems(streams);
 }
 inline int chunk2(bool hm, bool pe) { return Ring2::tile_elems(2 + (hm ? 1 : 0) + (pe ? 1 : 0)); }
-inline int chunk1_min(int K) { return chunk1(K, true, K == 1); }
+// No pass-1 tile is smaller: K (+1 with g_small) streams in 36 KB, or K + 1 in 45 KB.
+inline int chunk1_min(int K) { return Ring1::tile_elems(K + 1 + (K == 1 ? 1 : 0)); }
 inline int chunk2_min() { return chunk2(true, true); }
 
 struct Plan {
@@ -2071,7 +2080,7 @@ int run_reduce_k(int K, int n, const int64_t *numels, const Scalars &sc, int gri
                  Fill fill, void *mid_event, bool finish, TableCache *cache) {
     const int chunk = chunk1(K, RW, SS);
     int rc = launch_streaming<P1<KT>::NP>(k_reduce<KT, WM, RW, SS, PR>, n, numels, chunk,
-                                          Ring1::kThreads, Ring1::kSmemBytes, sc,
+                                          Ring1Of<RW>::kThreads, Ring1Of<RW>::kSmemBytes, sc,
                                           grid, s, fill, cache);
     if (rc) return rc;
     record(mid_event, s);
@@ -2134,6 +2143,7 @@ int tula_ags_chunk_elems(int pass, int streams) {
     if (streams < 1 || streams > TULA_MAX_K + 2) return TULA_ERR_ARG;
     if (pass == 1) return Ring1::tile_elems(streams);
     if (pass == 2 && streams <= 4) return Ring2::tile_elems(streams);
+    if (pass == 3) return Ring1W::tile_elems(streams);
     return TULA_ERR_ARG;
 }
 

@@ -40,7 +40,8 @@ def test_defaults_match_paper(lib):
 
 
 @pytest.mark.parametrize("pass_,stage_kb,streams", [(1, 36, s) for s in (1, 2, 3, 4, 9, 17, 18)]
-                         + [(2, 24, s) for s in (2, 3, 4)])
+                         + [(2, 24, s) for s in (2, 3, 4)]
+                         + [(3, 45, s) for s in (2, 3, 5, 9, 17)])
 def test_tile_fits_one_stage(lib, pass_, stage_kb, streams):
     C = T.tula_ags_chunk_elems(pass_, streams)
     stage = stage_kb * 1024
@@ -49,7 +50,7 @@ def test_tile_fits_one_stage(lib, pass_, stage_kb, streams):
 
 
 def test_tile_sizes_reject_bad_arguments(lib):
-    for pass_, streams in ((1, 0), (1, 19), (2, 0), (2, 5), (0, 2), (3, 2)):
+    for pass_, streams in ((1, 0), (1, 19), (2, 0), (2, 5), (0, 2), (3, 0), (3, 19), (4, 2)):
         assert T.lib().tula_ags_chunk_elems(pass_, streams) == T.TULA_ERR_ARG
 
 

@@ -28,11 +28,13 @@ def _built():
 
 def _ragged_pset(extra=(), K=None):
     """Empty, tiny and ragged tensors; with K, also sizes one below, at and one above a tile and
-    two tiles of either pass (the tile sizes the library uses for K replicas)."""
+    two tiles of every pass (the tile sizes the library uses for K replicas: pass 1, pass 2, and
+    pass 1 reading w)."""
     ps = W.ParamSet("ragged")
     sizes = [0, 1, 3, 4, 5, 63, 64, 65, 4095, CHUNK - 1, CHUNK, CHUNK + 1, 40000, 100003, *extra]
     if K is not None:
-        for t in (T.tula_ags_chunk_elems(1, K), T.tula_ags_chunk_elems(2, 3)):
+        for t in (T.tula_ags_chunk_elems(1, K), T.tula_ags_chunk_elems(2, 3),
+                  T.tula_ags_chunk_elems(3, K + 1)):
             sizes += [t - 1, t, t + 1, 2 * t + 1]
     for n in sizes:
         ps.add((n,), W.KIND_NORMAL)
@@ -413,14 +415,16 @@ def test_calls_back_to_back_on_one_workspace_and_stream(K):
         assert_f32_close(buf.m[p].reshape(-1).cpu().numpy(), pair.m_h[p], f"m[{p}]")
 
 
-def _extreme_pset(streams):
-    """Tensors of one element to several tiles (ragged tails) of a pass-1 tile of `streams`
-    streams, three times over, for per-tensor gradient factors spread over 46 decades."""
+def _extreme_pset(*tiles):
+    """Tensors of one element to several tiles (ragged tails) of each pass-1 tile given as
+    (pass, streams) -- pass 3 is pass 1 when it reads w -- three times over, for per-tensor
+    gradient factors spread over 46 decades."""
     ps = W.ParamSet("extremes")
-    t = T.tula_ags_chunk_elems(1, streams)
-    for _ in range(3):
-        for n in (1, 5, 64, 1000, t - 1, t + 3, 2 * t + 7, 40000):
-            ps.add((n,), W.KIND_NORMAL)
+    for pass_, streams in tiles:
+        t = T.tula_ags_chunk_elems(pass_, streams)
+        for _ in range(3):
+            for n in (1, 5, 64, 1000, t - 1, t + 3, 2 * t + 7, 40000):
+                ps.add((n,), W.KIND_NORMAL)
     return ps
 
 
@@ -436,7 +440,7 @@ def test_lars_steps_over_the_whole_float_range():
     """LARS steps take every pass-1 norm precisely.  Gradient factors from 1e-24 to 1e22: the
     squares of some tensors underflow or overflow fp32 (they go through fp64), the others are
     split exactly into float-float pairs; coefficients, norms and updates match the oracle."""
-    ps = _extreme_pset(3)
+    ps = _extreme_pset((3, 3))
     wl = _extreme_workload(97, ps)
     pair = Pair(wl, K=2, pset=ps, rule=T.TULA_RULE_LARS, lars_trust=0.01)
     pair.step(1, 1.0)
@@ -446,7 +450,7 @@ def test_lars_steps_over_the_whole_float_range():
 def test_update_scale_over_the_whole_float_range():
     """UpdateGradScale per tensor (precise norms of g_small and g_large) over the same range,
     with s_max out of the way: each scale within 2 ulp of the oracle's fp64 ratio."""
-    ps = _extreme_pset(2)
+    ps = _extreme_pset((1, 2))
     wl = _extreme_workload(105, ps)
     buf = W.allocate(wl, "cuda", K=2, pset=ps)
     W.fill_grads(buf, wl, step=1)
@@ -482,7 +486,7 @@ def test_default_steps_over_the_whole_float_range():
     tula_layer_stats, with gradient and weight factors from 1e-24 to 1e22: tiles whose fp32
     sums of squares would overflow, underflow, or hold only zeros are summed again with an exact
     power-of-two scaling; norms, |G|^2, Delta, the branch, w and m match the oracle."""
-    ps = _extreme_pset(2)
+    ps = _extreme_pset((1, 2), (3, 3))   # the step's pass 1, and tula_layer_stats' (reads w)
     wl = _extreme_workload(113, ps)
     pair = Pair(wl, K=2, pset=ps)
     _scale_weights(pair, 113)
@@ -510,7 +514,7 @@ def test_default_steps_over_the_whole_float_range():
 def test_default_steps_misaligned_over_the_whole_float_range(K):
     """The same range on misaligned tensors, where every element is loaded one by one (fp64
     squares), and with K = 1 and 4 (other tile sizes and stream counts)."""
-    ps = _extreme_pset(K if K > 1 else 1)
+    ps = _extreme_pset((1, K if K > 1 else 1))
     wl = _extreme_workload(121 + K, ps)
     for shift in (0, 1):
         pair = Pair(wl, K=K, pset=ps, align=1 if shift else 64, shift=shift)
