@@ -96,7 +96,7 @@ def job_throughput(params_per_rank: int, steps: int, world_size: int, t_max_ms: 
 LARS_TRUST = 1e-3  # trust coefficient of the LARS steps timed here
 # step kind -> (reads w in pass 1, refreshes the gradscale every step)
 STEP_KINDS = {"ags": (False, False), "refresh": (False, True), "lars": (True, False),
-              "update-scale": (False, False)}
+              "update-scale": (False, False), "sharded": (False, False)}
 
 
 def pass1_bytes_per_param(K: int, read_w: bool = False) -> int:
@@ -348,6 +348,9 @@ STEP_KIND_TEXT = {
     "refresh": "Algorithm 1 step that also refreshes the gradscale (UpdateGradScale, g_small = "
                "replica 0)",
     "lars": "LARS rule step (coefficient 0.001 |w| / |gbar|)",
+    "sharded": "Algorithm 1 step sharded over 2 ranks run one after the other on one GPU (pass 1 "
+               "of each shard, the shares of |G|^2 summed by an integer add on the GPU, then the "
+               "rest of each shard): the same results as the whole step",
 }
 
 
@@ -723,8 +726,80 @@ def run_update_scale(args, wl):
         "config": _config(wl, wl.pset, "update-scale"),
         "roofline": {"bound": "hbm", "kernel": "k_scale_elem (UpdateGradScale, element-wise)",
                      "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
-                     "peak_kind": peak_kind, "traffic": None,
+                     "peak_kind": peak_kind, "traffic": _ncu_traffic("k_scale_elem", wl.name, N),
                      "bytes_per_launch": scale_elem_bytes_per_param() * N, "ms_per_launch": ms},
+        "e2e": None, "gpu_launches": T.tula_ags_launch_count() - launches0, "clocks": clocks,
+    }), flush=True)
+
+
+def run_sharded(args, wl):
+    """An Algorithm 1 step sharded over two ranks, emulated on one GPU by running the shards one
+    after the other: tula_ags_shard_reduce on each half of the tensors, their shares of |G|^2
+    added as integers (the exchange), tula_ags_shard_update on each half.  One process; it
+    measures what sharding adds to a step (two passes per shard, the exchange) on the same
+    parameter set, not a multi-GPU rate."""
+    import torch
+
+    from paper_2603_18112_gb300 import build as B
+    from paper_2603_18112_gb300 import tula_ags as T
+    from paper_2603_18112_gb300 import workloads as W
+    if _dist()[0] > 1:
+        raise SystemExit("--step-kind sharded runs its ranks one after the other on one GPU")
+    if not B.LIB.exists():
+        B.build()
+    T.lib()
+    buf = W.allocate(wl, "cuda")
+    W.fill_state(buf, wl)
+    W.fill_grads(buf, wl, step=1)
+    K, n = wl.K, buf.pset.n_tensors
+    cut = n // 2 + 1
+    ranks = [T.AGSOptimizerStep(buf.w[lo:hi], [buf.g[k][lo:hi] for k in range(K)],
+                                buf.m[lo:hi], s_max=wl.smax)
+             for lo, hi in ((0, cut), (cut, n))]
+    shares = [r.new_g2_share() for r in ranks]
+    total = torch.zeros_like(shares[0])
+    stream = torch.cuda.Stream()
+    torch.cuda.synchronize()
+
+    def one_step(refresh=False):
+        for r, sh in zip(ranks, shares):
+            r.shard_reduce(wl.momentum, sh, refresh_scale=refresh, stream=stream)
+        torch.add(shares[0], shares[1], out=total)
+        for r in ranks:
+            r.shard_update(wl.lr, wl.momentum, wl.weight_decay, total, refresh_scale=refresh,
+                           stream=stream)
+
+    with torch.cuda.stream(stream):
+        for i in range(max(3, args.warmup)):
+            one_step(refresh=(i == 0 and K > 1))
+    stream.synchronize()
+    sampler = ClockSampler(0)
+    sampler.start()
+    launches0 = T.tula_ags_launch_count()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        t0.record(stream)
+        for _ in range(args.steps):
+            one_step()
+        t1.record(stream)
+    stream.synchronize()
+    clocks = sampler.stop()
+    ms = t0.elapsed_time(t1) / args.steps
+    N = buf.pset.n_params
+    peak, peak_kind = _peaks()
+    per = step_min_bytes_per_param(K, False)
+    gbs = per * N / (ms / 1e3) / 1e9
+    config = _config(wl, buf.pset, "sharded")
+    config["parallelism"] = "2 shards of whole tensors, run one after the other on one GPU"
+    print(json.dumps({
+        "metric": METRIC, "value": N / (ms / 1e3), "unit": UNIT, "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": config,
+        "roofline": {"bound": "hbm", "kernel": "the whole sharded step (both shards)",
+                     "achieved": gbs, "peak": peak, "unit": "GB/s", "frac": gbs / peak,
+                     "peak_kind": peak_kind, "traffic": None,
+                     "bytes_per_launch": per * N, "ms_per_launch": ms},
         "e2e": None, "gpu_launches": T.tula_ags_launch_count() - launches0, "clocks": clocks,
     }), flush=True)
 
@@ -737,6 +812,8 @@ def main():
         run_reference(args, wl)
     elif args.step_kind == "update-scale":
         run_update_scale(args, wl)
+    elif args.step_kind == "sharded":
+        run_sharded(args, wl)
     else:
         run_ours(args, wl)
 

@@ -30,7 +30,8 @@ def test_bytes_per_parameter(K):
 def test_step_kinds():
     # only LARS reads w in pass 1; only the refresh kind refreshes the gradscale every step
     assert bench.STEP_KINDS == {"ags": (False, False), "refresh": (False, True),
-                                "lars": (True, False), "update-scale": (False, False)}
+                                "lars": (True, False), "update-scale": (False, False),
+                                "sharded": (False, False)}
     assert set(bench.STEP_KIND_TEXT) == set(bench.STEP_KINDS)
 
 
