@@ -92,14 +92,16 @@ def test_rules(rule, gran, mom):
     assert pair.flags[:3] == [0, 1, 0]
 
 
-def test_many_tensors_span_several_launches():
-    """1000 tensors with K = 16 need several parameter blocks per pass."""
+@pytest.mark.parametrize("rule", [T.TULA_RULE_AGS, T.TULA_RULE_LARS])
+def test_many_tensors_span_several_launches(rule):
+    """1000 tensors with K = 16 need several parameter blocks per pass (LARS: pass 1 reading w,
+    through its own ring and tile size)."""
     rng = np.random.default_rng(5)
     ps = W.ParamSet("many")
     for n in rng.integers(1, 5000, size=1000):
         ps.add((int(n),), W.KIND_NORMAL)
     wl = W.workload("stress_k16", seed=31)
-    pair = Pair(wl, pset=ps)
+    pair = Pair(wl, pset=ps, rule=rule, lars_trust=0.01)
     before = T.tula_ags_launch_count()
     for i, mult in enumerate((1.0, 1.0)):
         pair.step(i + 1, mult, refresh=(i == 0))
