@@ -56,10 +56,14 @@ def test_resnet20_ten_steps():
 
 @pytest.mark.parametrize("K", [1, 2, 3, 4, 5, 8, 16])
 @pytest.mark.parametrize("shift", [0, 1])
-def test_ragged_shapes(K, shift):
-    """Tensors of 0..100003 elements (ragged chunk tails); shift=1 misaligns every tensor."""
+@pytest.mark.parametrize("rule", [T.TULA_RULE_AGS, T.TULA_RULE_LARS])
+def test_ragged_shapes(K, shift, rule):
+    """Tensors of 0..100003 elements (ragged chunk tails); shift=1 misaligns every tensor.  LARS
+    takes pass 1 through its own ring (w read), K = 3 and 5 through the kernel compiled for any
+    K."""
     wl = W.workload("stress_k4", seed=11 + K, factor_range=(1e-3, 1e1), zero_patterns=False)
-    pair = Pair(wl, K=K, align=1 if shift else 64, shift=shift, pset=_ragged_pset(K=K))
+    pair = Pair(wl, K=K, align=1 if shift else 64, shift=shift, pset=_ragged_pset(K=K), rule=rule,
+                lars_trust=0.01)
     # draw 1 twice (Delta = 0: scaled), then x2 (Delta = 3: unscaled), then a fresh draw
     for i, (seed_step, mult) in enumerate(((1, 1.0), (1, 1.0), (1, 2.0), (2, 1.0))):
         pair.step(seed_step, mult, refresh=(K > 1 and i == 0))
